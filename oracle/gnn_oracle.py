@@ -1,0 +1,129 @@
+"""Oracle: plain, slow, fp64 CPU evaluation of the interaction-network edge classifier.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path imports this module:
+only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may call it.  It shares no code with the CUDA path.
+
+What it computes (Section 2.1: space points in, candidate edges between them,
+the edge-classification step is an interaction network whose per-edge scores
+feed the connected-components step).  The paper cites the interaction network
+without writing out its equations, so the network below is the plain
+message-passing definition the benchmark specifies, evaluated in float64:
+
+    MLP(v)      = for each layer l: v <- ReLU(LayerNorm_l(W_l v + b_l))
+    LayerNorm   : mean and biased variance over the H features,
+                  gamma * (v - mean) / sqrt(var + eps) + beta
+    f_ij        = (x_j[0] - x_i[0], wrap(x_j[1] - x_i[1]))   for edge i -> j
+    h_j         = MLP_node_encoder(x_j);  e_ij = MLP_edge_encoder(f_ij)
+    repeat T times:
+        m_ij    = MLP_edge_network([h_i, h_j, e_ij]);  e_ij <- m_ij
+        a_j     = sum over edges (i -> j) of m_ij     (zero when j has no in-edge)
+        h_j     = MLP_node_network([h_j, a_j])
+    logit_ij    = w_o . MLP_edge_classifier([h_i, h_j, e_ij]) + b_o
+    score_ij    = 1 / (1 + exp(-logit_ij))
+
+Edge features use the input's precision: the phi difference of two float32
+features is rounded to float32 and the wrap into (-1, 1] (units of pi; exact
++-1 maps to +1) is decided on that float32 value, so the oracle and a float32
+kernel take the same wrap decision.
+
+Every routine works on plain numpy arrays; the matrix product, argsort and
+np.add.at are the only library primitives used.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+MLP_NAMES = ("node_encoder", "edge_encoder", "edge_network", "node_network", "edge_classifier")
+
+
+def layer_norm(v: np.ndarray, gamma: np.ndarray, beta: np.ndarray, eps: float) -> np.ndarray:
+    """LayerNorm over the last axis with biased variance and affine gamma, beta."""
+    mu = v.mean(axis=-1, keepdims=True)
+    var = ((v - mu) ** 2).mean(axis=-1, keepdims=True)
+    return gamma * (v - mu) / np.sqrt(var + eps) + beta
+
+
+def relu(v: np.ndarray) -> np.ndarray:
+    return np.maximum(v, 0.0)
+
+
+def mlp(v: np.ndarray, layers, eps: float) -> np.ndarray:
+    """Stack of Linear -> LayerNorm -> ReLU layers; `layers` = [(W [out,in], b, gamma, beta)]."""
+    v = np.asarray(v, dtype=np.float64)
+    for (W, b, g, be) in layers:
+        W = np.asarray(W, np.float64)
+        v = relu(layer_norm(v @ W.T + np.asarray(b, np.float64),
+                            np.asarray(g, np.float64), np.asarray(be, np.float64), eps))
+    return v
+
+
+def wrap_dphi_f32(d: np.ndarray) -> np.ndarray:
+    """Wrap float32 phi differences (units of pi) into (-1, 1], in float32."""
+    d = np.asarray(d, dtype=np.float32)
+    two = np.float32(2.0)
+    out = np.where(d > np.float32(1.0), d - two, d)
+    out = np.where(out <= np.float32(-1.0), out + two, out)
+    return out.astype(np.float32)
+
+
+def edge_features(x: np.ndarray, src: np.ndarray, dst: np.ndarray) -> np.ndarray:
+    """f_ij = (dr, dphi) for every edge i -> j, computed in float32 (see module doc)."""
+    x = np.asarray(x, dtype=np.float32)
+    dr = (x[dst, 0] - x[src, 0]).astype(np.float32)
+    dphi = wrap_dphi_f32((x[dst, 1] - x[src, 1]).astype(np.float32))
+    return np.stack([dr, dphi], axis=1)
+
+
+def csr_by_destination(src: np.ndarray, dst: np.ndarray, n_nodes: int):
+    """Destination-keyed CSR: edges stably sorted by destination (ties keep input
+    order).  Returns rowptr [N+1], src_sorted [E], perm [E] (sorted slot -> input id)."""
+    dst = np.asarray(dst, dtype=np.int64)
+    perm = np.argsort(dst, kind="stable")
+    counts = np.bincount(dst, minlength=n_nodes) if dst.size else np.zeros(n_nodes, np.int64)
+    rowptr = np.zeros(n_nodes + 1, dtype=np.int64)
+    rowptr[1:] = np.cumsum(counts)
+    return rowptr, np.asarray(src, np.int64)[perm], perm
+
+
+def aggregate(m: np.ndarray, dst: np.ndarray, n_nodes: int) -> np.ndarray:
+    """a_j = sum of the messages of all edges whose destination is j (0 if none)."""
+    a = np.zeros((n_nodes, m.shape[1]), dtype=np.float64)
+    np.add.at(a, np.asarray(dst, np.int64), m)
+    return a
+
+
+def sigmoid(z: np.ndarray) -> np.ndarray:
+    z = np.asarray(z, dtype=np.float64)
+    return np.where(z >= 0, 1.0 / (1.0 + np.exp(-np.abs(z))),
+                    np.exp(-np.abs(z)) / (1.0 + np.exp(-np.abs(z))))
+
+
+def forward(weights: dict, x: np.ndarray, edge_index: np.ndarray, n_iters: int,
+            eps: float = 1e-5, return_logits: bool = False, return_states: bool = False):
+    """Edge scores (input edge order) of the interaction network on one hit graph.
+
+    `weights` maps each MLP name to its [(W, b, gamma, beta)] layers, plus
+    'head_w' [H] and 'head_b' [1].  `edge_index` is [2, E] (row 0 source, row 1
+    destination).  Returns scores (and logits / final states on request)."""
+    x = np.asarray(x, dtype=np.float32)
+    src = np.asarray(edge_index[0], dtype=np.int64)
+    dst = np.asarray(edge_index[1], dtype=np.int64)
+    n_nodes = x.shape[0]
+    f = edge_features(x, src, dst).astype(np.float64)
+    h = mlp(x.astype(np.float64), weights["node_encoder"], eps)
+    e = mlp(f, weights["edge_encoder"], eps)
+    for _ in range(n_iters):
+        m = mlp(np.concatenate([h[src], h[dst], e], axis=1), weights["edge_network"], eps)
+        e = m
+        a = aggregate(m, dst, n_nodes)
+        h = mlp(np.concatenate([h, a], axis=1), weights["node_network"], eps)
+    c = mlp(np.concatenate([h[src], h[dst], e], axis=1), weights["edge_classifier"], eps)
+    logits = c @ np.asarray(weights["head_w"], np.float64) + float(np.asarray(weights["head_b"])[0])
+    scores = sigmoid(logits)
+    out = [scores]
+    if return_logits:
+        out.append(logits)
+    if return_states:
+        out.append({"h": h, "e": e})
+    return out[0] if len(out) == 1 else tuple(out)
