@@ -1,0 +1,146 @@
+/*
+ * gnn.h -- C ABI of the GB300 interaction-network edge classifier.
+ *
+ * The library scores candidate edges of a particle-detector hit graph with an
+ * interaction network, the edge-classification stage of the GNN tracking
+ * pipeline (paper Section 2.1: space points and the candidate edges built
+ * between them go in; the interaction network gives every edge a score that
+ * the connected-components step thresholds into track candidates).  The
+ * paper's service boundary takes a 2-D array of space points (rows) by raw
+ * features (columns) (Section 2.3); this ABI keeps that layout and adds the
+ * candidate edges, and returns one score per edge.
+ *
+ * Network (fp32 model; every MLP is L x [Linear -> LayerNorm -> ReLU]):
+ *   h_j  = MLP_node_encoder(x_j)            e_ij = MLP_edge_encoder(dr, dphi)
+ *   T times: m_ij = MLP_edge([h_i, h_j, e_ij]);  e_ij = m_ij
+ *            a_j  = sum over edges (i -> j) of m_ij
+ *            h_j  = MLP_node([h_j, a_j])
+ *   score_ij = sigmoid(w_o . MLP_classifier([h_i, h_j, e_ij]) + b_o)
+ * with dr = x_j[0] - x_i[0] and dphi = x_j[1] - x_i[1] wrapped into (-1, 1]
+ * (columns 0 and 1 hold r/1000 and phi/pi).
+ *
+ * Threading and streams: every call that takes a stream only enqueues work on
+ * it (no host synchronisation) unless stated otherwise.  A context is not
+ * safe for concurrent use from several streams or threads (it owns one
+ * workspace); use one context per stream.
+ *
+ * Return codes: GNN_OK (0) or a negative gnn_status_code.  Errors found on
+ * the host are returned at once; errors found by the kernels are recorded in
+ * the context's device error word and returned by gnn_status().
+ */
+#ifndef GNN_GB300_H
+#define GNN_GB300_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* gnn_stream_t; /* a cudaStream_t; NULL = legacy default stream */
+
+enum gnn_status_code {
+  GNN_OK = 0,
+  GNN_ERR_INVALID_ARG = -1,    /* null pointer, bad size or unsupported configuration */
+  GNN_ERR_BAD_WEIGHTS = -2,    /* weight blob: wrong magic/version/size or config mismatch */
+  GNN_ERR_OOM = -3,            /* device allocation failed */
+  GNN_ERR_CUDA = -4,           /* a CUDA runtime call or kernel launch failed */
+  GNN_ERR_INDEX_RANGE = -5,    /* device: an edge endpoint was outside [0, n_nodes) */
+  GNN_ERR_DEVICE_TIMEOUT = -6, /* device: a pipeline wait expired; results are invalid */
+};
+
+enum gnn_precision {
+  GNN_PRECISION_FP32 = 0,      /* fp32 weights and state; products as three bf16 pieces */
+  GNN_PRECISION_BF16 = 1,      /* reserved: bf16 weights and state (not built yet) */
+};
+
+/* Model configuration (must equal the blob header). */
+typedef struct gnn_config {
+  int32_t version;             /* must be 1 */
+  int32_t n_node_feat;         /* F_n: node feature columns, 2..16 (cols 0, 1 = r/1000, phi/pi) */
+  int32_t n_edge_feat;         /* must be 2: (dr, dphi) */
+  int32_t hidden;              /* H: 64 or 128 */
+  int32_t n_iters;             /* T: message-passing iterations, 0..64 */
+  int32_t mlp_layers;          /* L: Linear layers per MLP, 2..4 */
+  int32_t precision;           /* enum gnn_precision */
+  float ln_eps;                /* LayerNorm epsilon (1e-5) */
+} gnn_config;
+
+typedef struct gnn_ctx gnn_ctx;
+
+/*
+ * gnn_create -- build a context on the current CUDA device.
+ *
+ * weights_host: host pointer to a little-endian weight blob of weights_bytes
+ * bytes: a header of eight int32 (magic 0x57474E47, version 1, n_node_feat,
+ * n_edge_feat, hidden, n_iters, mlp_layers, precision), float32 ln_eps, int32
+ * reserved, int64 float count; then float32 arrays.  For each MLP in the order
+ * node_encoder, edge_encoder, edge_network, node_network, edge_classifier and
+ * each of its L layers: W [H, in] row-major, b [H], gamma [H], beta [H]
+ * (in = F_n, 2, 3H, 2H, 3H for layer 1, H afterwards; the 3H inputs are
+ * ordered [h_src, h_dst, e] and the 2H input [h, a]); then w_o [H] and b_o [1].
+ * The blob is copied and repacked; the caller may free it on return.
+ * On success *out receives the context (free with gnn_destroy).
+ * Errors: INVALID_ARG (null pointer, unsupported config), BAD_WEIGHTS, OOM,
+ * CUDA.  Synchronous.
+ */
+int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_bytes, gnn_ctx** out);
+
+/*
+ * gnn_reserve -- size the context's workspace for graphs up to max_nodes
+ * nodes and max_edges edges, so that later gnn_infer calls of that size
+ * allocate nothing.  Synchronous (device allocation).  Errors: INVALID_ARG,
+ * OOM.
+ */
+int gnn_reserve(gnn_ctx* ctx, int64_t max_nodes, int64_t max_edges);
+
+/*
+ * gnn_infer -- score every edge of one graph (a single event, or several
+ * events concatenated block-diagonally).
+ *
+ *   node_feats  device, float32 [n_nodes, n_node_feat] row-major, 16-byte aligned
+ *   edge_index  device, int32 [2, n_edges] row-major: row 0 = source ids,
+ *               row 1 = destination ids, any order; duplicates and
+ *               self-loops are legal
+ *   edge_scores device, float32 [n_edges]: score of edge k of the input order
+ *
+ * All three buffers are caller-owned and must stay valid until the stream
+ * reaches this work; the library never frees them.  n_edges == 0 is a no-op;
+ * n_nodes == 0 with n_edges > 0 and sizes above INT32_MAX - 1 are
+ * INVALID_ARG.  The workspace grows here (synchronous allocation) when the
+ * graph is larger than any earlier one; call gnn_reserve first to avoid it.
+ * An edge with an endpoint outside [0, n_nodes) gets a NaN score, takes no
+ * part in any aggregation, and makes gnn_status report INDEX_RANGE.
+ * Scores are deterministic: the same inputs give bitwise-identical outputs.
+ */
+int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
+              int64_t n_edges, float* edge_scores, gnn_stream_t stream);
+
+/*
+ * gnn_status -- synchronise `stream`, then return and clear the device error
+ * word of the context: GNN_OK, GNN_ERR_INDEX_RANGE, GNN_ERR_DEVICE_TIMEOUT or
+ * GNN_ERR_CUDA (a failed synchronisation).
+ */
+int gnn_status(gnn_ctx* ctx, gnn_stream_t stream);
+
+/* gnn_destroy -- synchronise the device work of ctx and free it. NULL is a no-op. */
+void gnn_destroy(gnn_ctx* ctx);
+
+/* gnn_error_string -- static text for a status code. */
+const char* gnn_error_string(int code);
+
+/*
+ * gnn_debug_copy -- test hook: copy an internal buffer of the last gnn_infer
+ * into caller device memory `dst` of at least `bytes` bytes (enqueued on
+ * `stream`).  which: 0 rowptr int32 [N+1], 1 perm int32 [E] (CSR slot ->
+ * input edge id), 2 src_sorted int32 [E], 3 node state h float32 [N, H],
+ * 4 edge state e float32 [E, H] in CSR order.  Errors: INVALID_ARG when the
+ * buffer is unknown or `bytes` is too small.
+ */
+int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GNN_GB300_H */

@@ -1,0 +1,124 @@
+"""ctypes binding of the C ABI in include/gnn.h (argument marshalling only).
+
+Device memory and streams come from PyTorch tensors; every step of the
+computation runs in the library's CUDA kernels."""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libgnn_gb300.so")
+_lib = None
+
+GNN_OK = 0
+ERRORS = {-1: "INVALID_ARG", -2: "BAD_WEIGHTS", -3: "OOM", -4: "CUDA", -5: "INDEX_RANGE",
+          -6: "DEVICE_TIMEOUT"}
+EXPORTED = ("gnn_create", "gnn_reserve", "gnn_infer", "gnn_status", "gnn_destroy",
+            "gnn_error_string", "gnn_debug_copy")
+
+
+class GnnError(RuntimeError):
+    def __init__(self, code: int, what: str = ""):
+        self.code = code
+        super().__init__(f"{what}: {ERRORS.get(code, code)} ({code})")
+
+
+class GnnConfig(ctypes.Structure):
+    _fields_ = [("version", ctypes.c_int32), ("n_node_feat", ctypes.c_int32),
+                ("n_edge_feat", ctypes.c_int32), ("hidden", ctypes.c_int32),
+                ("n_iters", ctypes.c_int32), ("mlp_layers", ctypes.c_int32),
+                ("precision", ctypes.c_int32), ("ln_eps", ctypes.c_float)]
+
+
+def load_library(path: str = LIB_PATH):
+    """Load the CUDA library; raises when it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"CUDA library not built ({path}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(path)
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+    lib.gnn_create.argtypes = [ctypes.POINTER(GnnConfig), vp, ctypes.c_size_t, ctypes.POINTER(vp)]
+    lib.gnn_create.restype = i32
+    lib.gnn_reserve.argtypes = [vp, i64, i64]
+    lib.gnn_reserve.restype = i32
+    lib.gnn_infer.argtypes = [vp, vp, vp, i64, i64, vp, vp]
+    lib.gnn_infer.restype = i32
+    lib.gnn_status.argtypes = [vp, vp]
+    lib.gnn_status.restype = i32
+    lib.gnn_destroy.argtypes = [vp]
+    lib.gnn_destroy.restype = None
+    lib.gnn_error_string.argtypes = [i32]
+    lib.gnn_error_string.restype = ctypes.c_char_p
+    lib.gnn_debug_copy.argtypes = [vp, i32, vp, ctypes.c_size_t, vp]
+    lib.gnn_debug_copy.restype = i32
+    _lib = lib
+    return lib
+
+
+def _stream_handle(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+class InteractionNetwork:
+    """One library context: a model (config + weight blob) on the current device."""
+
+    def __init__(self, model_cfg, blob: bytes):
+        self.lib = load_library()
+        self.cfg = model_cfg
+        c = GnnConfig(1, model_cfg.n_node_feat, model_cfg.n_edge_feat, model_cfg.hidden,
+                      model_cfg.n_iters, model_cfg.mlp_layers, model_cfg.precision, model_cfg.ln_eps)
+        buf = ctypes.create_string_buffer(blob, len(blob))
+        h = ctypes.c_void_p()
+        rc = self.lib.gnn_create(ctypes.byref(c), buf, len(blob), ctypes.byref(h))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_create")
+        self.handle = h
+
+    def reserve(self, n_nodes: int, n_edges: int):
+        rc = self.lib.gnn_reserve(self.handle, n_nodes, n_edges)
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_reserve")
+
+    def infer(self, x, edge_index, scores=None, stream=None):
+        """x: cuda float32 [N, F_n]; edge_index: cuda int32 [2, E]; returns cuda float32 [E]."""
+        import torch
+        assert x.is_cuda and x.dtype == torch.float32 and x.is_contiguous()
+        assert edge_index.is_cuda and edge_index.dtype == torch.int32 and edge_index.is_contiguous()
+        E = edge_index.shape[1]
+        if scores is None:
+            scores = torch.empty(E, dtype=torch.float32, device=x.device)
+        rc = self.lib.gnn_infer(self.handle, ctypes.c_void_p(x.data_ptr()),
+                                ctypes.c_void_p(edge_index.data_ptr()), x.shape[0], E,
+                                ctypes.c_void_p(scores.data_ptr()), _stream_handle(stream))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_infer")
+        return scores
+
+    def status(self, stream=None) -> int:
+        return self.lib.gnn_status(self.handle, _stream_handle(stream))
+
+    def debug_copy(self, which: int, shape, dtype, stream=None):
+        import torch
+        out = torch.empty(shape, dtype=dtype, device="cuda")
+        rc = self.lib.gnn_debug_copy(self.handle, which, ctypes.c_void_p(out.data_ptr()),
+                                     out.numel() * out.element_size(), _stream_handle(stream))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_debug_copy")
+        return out
+
+    def close(self):
+        if getattr(self, "handle", None):
+            self.lib.gnn_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,139 @@
+// Destination-keyed CSR of the candidate edges, built on the device.
+//
+// The message-passing step sums every edge's message into its destination
+// node.  Sorting the edges by destination turns that sum into a contiguous
+// segment per node, read in a fixed order (deterministic, no float atomics),
+// and lets the edge kernels stream the per-edge state in that order.
+//
+// Steps: validate endpoints and form keys (key = dst, or n_nodes for an edge
+// with an endpoint out of range), stable LSD radix sort of (key, input id)
+// with 8-bit digits, then gather the sources in sorted order and mark the
+// first slot of every node (rowptr).  A stable sort of keys that only differ
+// in input id gives the unique order "by destination, then input id".
+#pragma once
+#include <cstdint>
+#include "ptx.cuh"
+
+namespace gnn {
+
+constexpr int kRadixThreads = 256;
+constexpr int kRadixRounds = 16;
+constexpr int kRadixTile = kRadixThreads * kRadixRounds;   // elements per tile
+
+// K0: endpoint validation and sort keys.
+__global__ void csr_keys_kernel(const int32_t* __restrict__ ei, int n_edges, int n_nodes,
+                                int* __restrict__ keys, int* __restrict__ vals,
+                                int* __restrict__ src_clamped, uint32_t* err) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= n_edges) return;
+  const int s = ei[k];
+  const int d = ei[(size_t)n_edges + k];
+  const bool ok = (s >= 0) & (s < n_nodes) & (d >= 0) & (d < n_nodes);
+  keys[k] = ok ? d : n_nodes;
+  vals[k] = k;
+  src_clamped[k] = ok ? s : 0;
+  if (!ok) atomicOr(err, DEV_ERR_INDEX_RANGE);
+}
+
+// Per-tile digit histogram: hist[digit * n_tiles + tile].
+__global__ void radix_count_kernel(const int* __restrict__ keys, int n, int shift, int n_tiles,
+                                   int* __restrict__ hist) {
+  __shared__ int cnt[256];
+  cnt[threadIdx.x] = 0;
+  __syncthreads();
+  const int base = blockIdx.x * kRadixTile;
+  for (int i = threadIdx.x; i < kRadixTile; i += kRadixThreads) {
+    const int idx = base + i;
+    if (idx < n) atomicAdd(&cnt[(keys[idx] >> shift) & 255], 1);
+  }
+  __syncthreads();
+  hist[threadIdx.x * n_tiles + blockIdx.x] = cnt[threadIdx.x];
+}
+
+// In-place exclusive scan of n ints with one block of 1024 threads.
+__global__ void exclusive_scan_kernel(int* __restrict__ data, int n) {
+  __shared__ int part[1024];
+  const int t = threadIdx.x;
+  const int per = (n + 1023) / 1024;
+  const int b = t * per, e = min(n, b + per);
+  int s = 0;
+  for (int i = b; i < e; ++i) s += data[i];
+  part[t] = s;
+  __syncthreads();
+  for (int off = 1; off < 1024; off <<= 1) {      // Hillis-Steele inclusive scan
+    const int v = (t >= off) ? part[t - off] : 0;
+    __syncthreads();
+    part[t] += v;
+    __syncthreads();
+  }
+  int run = part[t] - s;                           // exclusive prefix of this chunk
+  for (int i = b; i < e; ++i) { const int v = data[i]; data[i] = run; run += v; }
+}
+
+// Stable scatter of one radix pass.  Elements of a tile are ranked in input
+// order: round r handles elements [r*256, r*256+256); within a warp the rank
+// among equal digits comes from __match_any_sync, across warps from per-warp
+// digit counts, across rounds from a running per-digit counter.
+__global__ void radix_scatter_kernel(const int* __restrict__ keys_in, const int* __restrict__ vals_in,
+                                     int* __restrict__ keys_out, int* __restrict__ vals_out, int n,
+                                     int shift, int n_tiles, const int* __restrict__ offs) {
+  __shared__ int run[256];
+  __shared__ int wcnt[kRadixThreads / 32][256];
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  run[t] = offs[t * n_tiles + blockIdx.x];
+  const int base = blockIdx.x * kRadixTile;
+  const unsigned lt_mask = (1u << lane) - 1u;
+  for (int r = 0; r < kRadixRounds; ++r) {
+    const int idx = base + r * kRadixThreads + t;
+    const bool has = idx < n;
+    const int key = has ? keys_in[idx] : 0;
+    const int val = has ? vals_in[idx] : 0;
+    const int dig = has ? ((key >> shift) & 255) : 256;
+#pragma unroll
+    for (int w = 0; w < kRadixThreads / 32; ++w) wcnt[w][t] = 0;
+    __syncthreads();
+    const unsigned peers = __match_any_sync(0xffffffffu, dig);
+    const int rank = __popc(peers & lt_mask);
+    if (has && rank == 0) wcnt[warp][dig] = __popc(peers);
+    __syncthreads();
+    if (has) {
+      int pos = run[dig] + rank;
+      for (int w = 0; w < warp; ++w) pos += wcnt[w][dig];
+      keys_out[pos] = key;
+      vals_out[pos] = val;
+    }
+    __syncthreads();
+    int add = 0;
+#pragma unroll
+    for (int w = 0; w < kRadixThreads / 32; ++w) add += wcnt[w][t];
+    run[t] += add;
+    __syncthreads();
+  }
+}
+
+// Sorted order -> perm, src_sorted, dst_sorted (clamped for invalid edges).
+__global__ void csr_gather_kernel(const int* __restrict__ keys_sorted, const int* __restrict__ vals_sorted,
+                                  const int* __restrict__ src_clamped, int n_edges, int n_nodes,
+                                  int* __restrict__ perm, int* __restrict__ src_sorted,
+                                  int* __restrict__ dst_sorted) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= n_edges) return;
+  const int id = vals_sorted[k];
+  const int key = keys_sorted[k];
+  perm[k] = id;
+  src_sorted[k] = src_clamped[id];
+  dst_sorted[k] = key < n_nodes ? key : 0;
+}
+
+// rowptr[j] = first sorted slot whose key >= j, for j in [0, n_nodes].
+__global__ void csr_rowptr_kernel(const int* __restrict__ keys_sorted, int n_edges, int n_nodes,
+                                  int* __restrict__ rowptr) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k > n_edges) return;
+  const int prev = (k == 0) ? -1 : keys_sorted[k - 1];
+  const int cur = (k == n_edges) ? n_nodes + 1 : keys_sorted[k];
+  const int hi = min(cur, n_nodes);
+  for (int j = prev + 1; j <= hi; ++j) rowptr[j] = k;
+}
+
+}  // namespace gnn

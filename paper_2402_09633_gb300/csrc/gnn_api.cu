@@ -1,0 +1,455 @@
+// C ABI and host orchestration of the interaction-network edge classifier.
+//
+// gnn_create parses the weight blob and repacks every H x H weight block into
+// the layout the tensor-core kernels read straight into shared memory
+// (bf16 hi and lo parts, K-major rows of 128 bytes, 128-byte swizzle).  The
+// first Linear layer of the edge network and of the classifier acts on
+// [h_src, h_dst, e]; it is split into three H x H blocks W_s, W_d, W_e so that
+//   W1 [h_src; h_dst; e] + b1 = (W_s h_src) + (W_d h_dst + b1) + W_e e,
+// where the two node terms are computed once per node (projections P_s, P_d)
+// instead of once per edge.  The node network's first layer on [h, a] is
+// split the same way into W_h and W_a.
+//
+// gnn_infer enqueues: CSR build (validate, radix sort by destination, gather,
+// row pointers) -> node encoder (+ projections) -> edge encoder -> T x (edge
+// update, node update with aggregation + projections) -> classifier.
+#include <cuda_runtime.h>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/gnn.h"
+#include "csr.cuh"
+#include "mlp_tiles.cuh"
+
+using namespace gnn;
+
+namespace {
+
+constexpr uint32_t kBlobMagic = 0x57474E47u;
+constexpr int kHeaderBytes = 8 * 4 + 4 + 4 + 8;
+
+struct Layer { const float* W; const float* b; const float* g; const float* be; int in; };
+
+enum Mlp { NODE_ENC = 0, EDGE_ENC = 1, EDGE_NET = 2, NODE_NET = 3, CLASSIFIER = 4, N_MLP = 5 };
+
+struct KernelPlan {          // job list and parameter vectors of one tile-kernel launch
+  int n_jobs = 0;
+  int job_mat[kMaxJobs] = {0};
+  int job_acc[kMaxJobs] = {0};
+  std::vector<float> vecs;
+  float* d_vecs = nullptr;
+};
+
+}  // namespace
+
+struct gnn_ctx {
+  gnn_config cfg;
+  int device = 0;
+  int n_sm = 0;
+  uint8_t* d_mats = nullptr;       // packed weight matrices
+  uint32_t mat_bytes = 0;
+  // plans: 0 node enc -> edge net, 1 node enc -> classifier, 2 edge enc,
+  //        3 edge update, 4 node update -> edge net, 5 node update -> classifier, 6 classifier
+  KernelPlan plan[7];
+  uint32_t* d_err = nullptr;
+  // workspace
+  void* ws = nullptr;
+  int64_t cap_nodes = -1, cap_edges = -1;
+  int *keys_a = nullptr, *keys_b = nullptr, *vals_a = nullptr, *vals_b = nullptr, *src_c = nullptr;
+  int *hist = nullptr, *perm = nullptr, *src_sorted = nullptr, *dst_sorted = nullptr, *rowptr = nullptr;
+  int* key_sorted = nullptr;
+  float *e = nullptr, *h = nullptr, *ps = nullptr, *pd = nullptr;
+  int64_t last_nodes = 0, last_edges = 0;
+};
+
+namespace {
+
+inline uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7F800000u) == 0x7F800000u) return (uint16_t)((u >> 16) | ((u & 0xFFFFu) ? 0x40u : 0u));
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+inline float bf16_to_f32(uint16_t h) {
+  uint32_t u = (uint32_t)h << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+// Byte offset of element (n, k) of an H x H block in the K-major, 128-byte
+// swizzled layout: 64-column chunks, 8-row atoms of 1024 bytes, 16-byte units
+// of a row permuted by XOR with the row index inside the atom.
+inline size_t swizzled_offset(int H, int n, int k) {
+  const int kc = k / 64, kk = k % 64;
+  return (size_t)kc * (H * 128) + (size_t)(n / 8) * 1024 + (n % 8) * 128 +
+         (((kk / 8) ^ (n % 8)) * 16) + (kk % 8) * 2;
+}
+
+// Pack columns [col0, col0+H) of W [H, ld] into hi/lo bf16 parts.
+void pack_block(const float* W, int ld, int col0, int H, uint8_t* out) {
+  const size_t part = (size_t)H * H * 2;
+  for (int n = 0; n < H; ++n)
+    for (int k = 0; k < H; ++k) {
+      const float v = W[(size_t)n * ld + col0 + k];
+      const uint16_t hi = f32_to_bf16_rne(v);
+      const uint16_t lo = f32_to_bf16_rne(v - bf16_to_f32(hi));
+      const size_t off = swizzled_offset(H, n, k);
+      std::memcpy(out + off, &hi, 2);
+      std::memcpy(out + part + off, &lo, 2);
+    }
+}
+
+void push(std::vector<float>& v, const float* p, size_t n) { v.insert(v.end(), p, p + n); }
+
+int cuda_fail(cudaError_t e) {
+  (void)cudaGetLastError();
+  return e == cudaErrorMemoryAllocation ? GNN_ERR_OOM : GNN_ERR_CUDA;
+}
+
+template <TileKind K, int H>
+cudaError_t set_smem_attr() {
+  return cudaFuncSetAttribute(mlp_tile_kernel<K, H>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              227 * 1024);
+}
+
+template <int H>
+cudaError_t set_all_attrs() {
+  cudaError_t e;
+  if ((e = set_smem_attr<TileKind::NodeEncoder, H>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::EdgeEncoder, H>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::EdgeUpdate, H>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::NodeUpdate, H>()) != cudaSuccess) return e;
+  return set_smem_attr<TileKind::Classifier, H>();
+}
+
+template <TileKind K, int H>
+void launch_tile(const gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st) {
+  p.n_jobs = pl.n_jobs;
+  for (int j = 0; j < kMaxJobs; ++j) { p.job_mat[j] = pl.job_mat[j]; p.job_acc[j] = pl.job_acc[j]; }
+  p.vecs = pl.d_vecs;
+  p.n_vec_floats = (int)pl.vecs.size();
+  p.wmats = c->d_mats;
+  p.mat_bytes = c->mat_bytes;
+  p.n_tiles = (p.n_rows + kTileRows - 1) / kTileRows;
+  if (p.n_tiles == 0) return;
+  uint32_t smem = tile_smem_bytes<H>(p.n_vec_floats);
+  if (smem < 120 * 1024) smem = 120 * 1024;           // one CTA per SM (it owns the TMEM)
+  const int pairs = (p.n_tiles + 1) / 2;
+  const int grid = pairs < c->n_sm ? pairs : c->n_sm;
+  mlp_tile_kernel<K, H><<<grid, kThreads, smem, st>>>(p);
+}
+
+template <int H>
+int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStream_t st) {
+  TileParams p{};
+  p.n_nodes = N;
+  p.n_layers = c->cfg.mlp_layers;
+  p.eps = c->cfg.ln_eps;
+  p.x = x;
+  p.x_stride = c->cfg.n_node_feat;
+  p.src_sorted = c->src_sorted;
+  p.dst_sorted = c->dst_sorted;
+  p.key_sorted = c->key_sorted;
+  p.perm = c->perm;
+  p.rowptr = c->rowptr;
+  p.e = c->e; p.h = c->h; p.ps = c->ps; p.pd = c->pd;
+  p.scores = scores;
+  p.err = c->d_err;
+  const int T = c->cfg.n_iters;
+
+  TileParams pn = p; pn.n_rows = N; pn.n_feat = c->cfg.n_node_feat;
+  launch_tile<TileKind::NodeEncoder, H>(c, c->plan[T > 0 ? 0 : 1], pn, st);
+  TileParams pe = p; pe.n_rows = E; pe.n_feat = 2;
+  launch_tile<TileKind::EdgeEncoder, H>(c, c->plan[2], pe, st);
+  for (int t = 1; t <= T; ++t) {
+    launch_tile<TileKind::EdgeUpdate, H>(c, c->plan[3], pe, st);
+    launch_tile<TileKind::NodeUpdate, H>(c, c->plan[t < T ? 4 : 5], pn, st);
+  }
+  launch_tile<TileKind::Classifier, H>(c, c->plan[6], pe, st);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
+
+void free_workspace(gnn_ctx* c) {
+  if (c->ws) cudaFree(c->ws);
+  c->ws = nullptr;
+  c->cap_nodes = c->cap_edges = -1;
+}
+
+int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
+  if (N <= c->cap_nodes && E <= c->cap_edges) return GNN_OK;
+  const int64_t n = N > c->cap_nodes ? N : c->cap_nodes;
+  const int64_t e = E > c->cap_edges ? E : c->cap_edges;
+  const int64_t H = c->cfg.hidden;
+  const int64_t rs_tiles = (e + kRadixTile - 1) / kRadixTile;
+  auto al = [](int64_t b) { return (b + 255) & ~int64_t(255); };
+  const int64_t sz_e_int = al(4 * (e > 0 ? e : 1));
+  const int64_t total = 8 * sz_e_int + al(4 * 256 * (rs_tiles > 0 ? rs_tiles : 1)) + al(4 * (n + 1)) +
+                        al(4 * e * H) + 3 * al(4 * n * H);
+  free_workspace(c);
+  void* ws = nullptr;
+  cudaError_t err = cudaMalloc(&ws, (size_t)total);
+  if (err != cudaSuccess) return cuda_fail(err);
+  c->ws = ws;
+  uint8_t* q = (uint8_t*)ws;
+  auto take = [&](int64_t bytes) { uint8_t* r = q; q += al(bytes); return r; };
+  c->keys_a = (int*)take(4 * e); c->keys_b = (int*)take(4 * e);
+  c->vals_a = (int*)take(4 * e); c->vals_b = (int*)take(4 * e);
+  c->src_c = (int*)take(4 * e); c->perm = (int*)take(4 * e);
+  c->src_sorted = (int*)take(4 * e); c->dst_sorted = (int*)take(4 * e);
+  c->hist = (int*)take(4 * 256 * (rs_tiles > 0 ? rs_tiles : 1));
+  c->rowptr = (int*)take(4 * (n + 1));
+  c->e = (float*)take(4 * e * H);
+  c->h = (float*)take(4 * n * H);
+  c->ps = (float*)take(4 * n * H);
+  c->pd = (float*)take(4 * n * H);
+  c->cap_nodes = n;
+  c->cap_edges = e;
+  return GNN_OK;
+}
+
+int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
+  const int tb = 256;
+  csr_keys_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(ei, E, N, c->keys_a, c->vals_a, c->src_c, c->d_err);
+  int bits = 0;
+  while (bits < 31 && (N >> bits) != 0) ++bits;        // keys lie in [0, N]
+  if (bits == 0) bits = 1;
+  const int passes = (bits + 7) / 8;
+  const int tiles = (E + kRadixTile - 1) / kRadixTile;
+  int *kin = c->keys_a, *vin = c->vals_a, *kout = c->keys_b, *vout = c->vals_b;
+  for (int ps = 0; ps < passes; ++ps) {
+    const int shift = 8 * ps;
+    radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, E, shift, tiles, c->hist);
+    exclusive_scan_kernel<<<1, 1024, 0, st>>>(c->hist, 256 * tiles);
+    radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, E, shift, tiles, c->hist);
+    int* t = kin; kin = kout; kout = t;
+    t = vin; vin = vout; vout = t;
+  }
+  c->key_sorted = kin;
+  csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, c->src_c, E, N, c->perm, c->src_sorted,
+                                                     c->dst_sorted);
+  csr_rowptr_kernel<<<(E + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, c->rowptr);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* gnn_error_string(int code) {
+  switch (code) {
+    case GNN_OK: return "ok";
+    case GNN_ERR_INVALID_ARG: return "invalid argument";
+    case GNN_ERR_BAD_WEIGHTS: return "bad weight blob";
+    case GNN_ERR_OOM: return "device out of memory";
+    case GNN_ERR_CUDA: return "CUDA error";
+    case GNN_ERR_INDEX_RANGE: return "edge endpoint out of range";
+    case GNN_ERR_DEVICE_TIMEOUT: return "device pipeline wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_bytes, gnn_ctx** out) {
+  if (!cfg || !weights_host || !out) return GNN_ERR_INVALID_ARG;
+  *out = nullptr;
+  const int H = cfg->hidden, L = cfg->mlp_layers, Fn = cfg->n_node_feat;
+  if (cfg->version != 1 || (H != 64 && H != 128) || L < 2 || L > 4 || Fn < 2 || Fn > 16 ||
+      cfg->n_edge_feat != 2 || cfg->n_iters < 0 || cfg->n_iters > 64 ||
+      cfg->precision != GNN_PRECISION_FP32 || !(cfg->ln_eps > 0.f))
+    return GNN_ERR_INVALID_ARG;
+  if (weights_bytes < (size_t)kHeaderBytes) return GNN_ERR_BAD_WEIGHTS;
+  const uint8_t* blob = (const uint8_t*)weights_host;
+  int32_t hdr[8];
+  float eps;
+  int64_t n_floats;
+  std::memcpy(hdr, blob, 32);
+  std::memcpy(&eps, blob + 32, 4);
+  std::memcpy(&n_floats, blob + 40, 8);
+  if ((uint32_t)hdr[0] != kBlobMagic || hdr[1] != 1 || hdr[2] != Fn || hdr[3] != 2 || hdr[4] != H ||
+      hdr[5] != cfg->n_iters || hdr[6] != L || hdr[7] != cfg->precision || eps != cfg->ln_eps)
+    return GNN_ERR_BAD_WEIGHTS;
+  const int in1[N_MLP] = {Fn, 2, 3 * H, 2 * H, 3 * H};
+  int64_t want = H + 1;
+  for (int m = 0; m < N_MLP; ++m) want += (int64_t)H * in1[m] + 3 * H + (int64_t)(L - 1) * (H * H + 3 * H);
+  if (n_floats != want || weights_bytes != (size_t)kHeaderBytes + 4 * (size_t)want) return GNN_ERR_BAD_WEIGHTS;
+
+  // locate arrays
+  const float* f = (const float*)(blob + kHeaderBytes);
+  Layer lay[N_MLP][4];
+  for (int m = 0; m < N_MLP; ++m)
+    for (int l = 0; l < L; ++l) {
+      const int in = l == 0 ? in1[m] : H;
+      lay[m][l] = {f, f + (size_t)H * in, f + (size_t)H * in + H, f + (size_t)H * in + 2 * H, in};
+      f += (size_t)H * in + 3 * H;
+    }
+  const float* head_w = f;
+  const float* head_b = f + H;
+
+  gnn_ctx* c = new (std::nothrow) gnn_ctx();
+  if (!c) return GNN_ERR_OOM;
+  c->cfg = *cfg;
+  cudaError_t err = cudaGetDevice(&c->device);
+  if (err == cudaSuccess) err = cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
+  if (err == cudaSuccess) err = (H == 128) ? set_all_attrs<128>() : set_all_attrs<64>();
+  if (err != cudaSuccess) { delete c; return cuda_fail(err); }
+
+  // matrices
+  std::vector<std::pair<const Layer*, int>> mats;   // (layer, column offset)
+  auto add_mat = [&](const Layer* ly, int col0) { mats.push_back({ly, col0}); return (int)mats.size() - 1; };
+  const int en_s = add_mat(&lay[EDGE_NET][0], 0), en_d = add_mat(&lay[EDGE_NET][0], H),
+            en_e = add_mat(&lay[EDGE_NET][0], 2 * H);
+  const int cl_s = add_mat(&lay[CLASSIFIER][0], 0), cl_d = add_mat(&lay[CLASSIFIER][0], H),
+            cl_e = add_mat(&lay[CLASSIFIER][0], 2 * H);
+  const int nn_h = add_mat(&lay[NODE_NET][0], 0), nn_a = add_mat(&lay[NODE_NET][0], H);
+  int deep[N_MLP][4];
+  for (int m = 0; m < N_MLP; ++m)
+    for (int l = 1; l < L; ++l) deep[m][l] = add_mat(&lay[m][l], 0);
+  c->mat_bytes = 2u * H * H * 2u;
+  std::vector<uint8_t> packed((size_t)c->mat_bytes * mats.size());
+  for (size_t i = 0; i < mats.size(); ++i)
+    pack_block(mats[i].first->W, mats[i].first->in, mats[i].second, H, packed.data() + i * c->mat_bytes);
+
+  // kernel plans
+  auto jobs = [](KernelPlan& pl, std::initializer_list<int> ids, int acc_mask = 0) {
+    pl.n_jobs = 0;
+    for (int id : ids) { pl.job_acc[pl.n_jobs] = (acc_mask >> pl.n_jobs) & 1; pl.job_mat[pl.n_jobs++] = id; }
+  };
+  auto add_deep = [&](KernelPlan& pl, int m) {
+    for (int l = 1; l < L; ++l) { pl.job_acc[pl.n_jobs] = 0; pl.job_mat[pl.n_jobs++] = deep[m][l]; }
+  };
+  auto bgb = [&](std::vector<float>& v, int m, int l0) {
+    for (int l = l0; l < L; ++l) { push(v, lay[m][l].b, H); push(v, lay[m][l].g, H); push(v, lay[m][l].be, H); }
+  };
+  for (int target = 0; target < 2; ++target) {           // node encoder -> edge net / classifier
+    KernelPlan& pl = c->plan[target];
+    pl.n_jobs = 0;
+    add_deep(pl, NODE_ENC);
+    pl.job_mat[pl.n_jobs++] = target == 0 ? en_s : cl_s;
+    pl.job_mat[pl.n_jobs++] = target == 0 ? en_d : cl_d;
+    push(pl.vecs, lay[NODE_ENC][0].W, (size_t)H * Fn);
+    bgb(pl.vecs, NODE_ENC, 0);
+    push(pl.vecs, lay[target == 0 ? EDGE_NET : CLASSIFIER][0].b, H);
+  }
+  {  // edge encoder
+    KernelPlan& pl = c->plan[2];
+    pl.n_jobs = 0;
+    add_deep(pl, EDGE_ENC);
+    push(pl.vecs, lay[EDGE_ENC][0].W, (size_t)H * 2);
+    bgb(pl.vecs, EDGE_ENC, 0);
+  }
+  {  // edge update
+    KernelPlan& pl = c->plan[3];
+    jobs(pl, {en_e});
+    add_deep(pl, EDGE_NET);
+    push(pl.vecs, lay[EDGE_NET][0].g, H);
+    push(pl.vecs, lay[EDGE_NET][0].be, H);
+    bgb(pl.vecs, EDGE_NET, 1);
+  }
+  for (int target = 0; target < 2; ++target) {           // node update -> edge net / classifier
+    KernelPlan& pl = c->plan[4 + target];
+    jobs(pl, {nn_h, nn_a}, 0b10);
+    add_deep(pl, NODE_NET);
+    pl.job_acc[pl.n_jobs] = 0; pl.job_mat[pl.n_jobs++] = target == 0 ? en_s : cl_s;
+    pl.job_acc[pl.n_jobs] = 0; pl.job_mat[pl.n_jobs++] = target == 0 ? en_d : cl_d;
+    bgb(pl.vecs, NODE_NET, 0);
+    push(pl.vecs, lay[target == 0 ? EDGE_NET : CLASSIFIER][0].b, H);
+  }
+  {  // classifier
+    KernelPlan& pl = c->plan[6];
+    jobs(pl, {cl_e});
+    add_deep(pl, CLASSIFIER);
+    push(pl.vecs, lay[CLASSIFIER][0].g, H);
+    push(pl.vecs, lay[CLASSIFIER][0].be, H);
+    bgb(pl.vecs, CLASSIFIER, 1);
+    push(pl.vecs, head_w, H);
+    push(pl.vecs, head_b, 1);
+  }
+
+  for (int i = 0; i < 7; ++i) c->plan[i].vecs.resize(padded_vec_floats((int)c->plan[i].vecs.size()), 0.f);
+  err = cudaMalloc(&c->d_mats, packed.size());
+  if (err == cudaSuccess) err = cudaMemcpy(c->d_mats, packed.data(), packed.size(), cudaMemcpyHostToDevice);
+  for (int i = 0; i < 7 && err == cudaSuccess; ++i) {
+    err = cudaMalloc(&c->plan[i].d_vecs, c->plan[i].vecs.size() * 4);
+    if (err == cudaSuccess)
+      err = cudaMemcpy(c->plan[i].d_vecs, c->plan[i].vecs.data(), c->plan[i].vecs.size() * 4, cudaMemcpyHostToDevice);
+  }
+  if (err == cudaSuccess) err = cudaMalloc(&c->d_err, 4);
+  if (err == cudaSuccess) err = cudaMemset(c->d_err, 0, 4);
+  if (err != cudaSuccess) { gnn_destroy(c); return cuda_fail(err); }
+  *out = c;
+  return GNN_OK;
+}
+
+int gnn_reserve(gnn_ctx* ctx, int64_t max_nodes, int64_t max_edges) {
+  if (!ctx || max_nodes < 0 || max_edges < 0 || max_nodes >= INT32_MAX || max_edges >= INT32_MAX)
+    return GNN_ERR_INVALID_ARG;
+  return ensure_workspace(ctx, max_nodes, max_edges);
+}
+
+int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
+              int64_t n_edges, float* edge_scores, gnn_stream_t stream) {
+  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX)
+    return GNN_ERR_INVALID_ARG;
+  if (n_edges == 0) return GNN_OK;
+  if (n_nodes == 0 || !node_feats || !edge_index || !edge_scores) return GNN_ERR_INVALID_ARG;
+  int rc = ensure_workspace(ctx, n_nodes, n_edges);
+  if (rc != GNN_OK) return rc;
+  cudaStream_t st = (cudaStream_t)stream;
+  const int N = (int)n_nodes, E = (int)n_edges;
+  rc = build_csr(ctx, edge_index, N, E, st);
+  if (rc != GNN_OK) return rc;
+  ctx->last_nodes = N;
+  ctx->last_edges = E;
+  return ctx->cfg.hidden == 128 ? run_network<128>(ctx, node_feats, N, E, edge_scores, st)
+                                : run_network<64>(ctx, node_feats, N, E, edge_scores, st);
+}
+
+int gnn_status(gnn_ctx* ctx, gnn_stream_t stream) {
+  if (!ctx) return GNN_ERR_INVALID_ARG;
+  cudaError_t err = cudaStreamSynchronize((cudaStream_t)stream);
+  if (err != cudaSuccess) return cuda_fail(err);
+  uint32_t word = 0;
+  err = cudaMemcpy(&word, ctx->d_err, 4, cudaMemcpyDeviceToHost);
+  if (err == cudaSuccess) err = cudaMemset(ctx->d_err, 0, 4);
+  if (err != cudaSuccess) return cuda_fail(err);
+  if (word & DEV_ERR_TIMEOUT) return GNN_ERR_DEVICE_TIMEOUT;
+  if (word & DEV_ERR_INDEX_RANGE) return GNN_ERR_INDEX_RANGE;
+  return GNN_OK;
+}
+
+void gnn_destroy(gnn_ctx* ctx) {
+  if (!ctx) return;
+  cudaDeviceSynchronize();
+  free_workspace(ctx);
+  if (ctx->d_mats) cudaFree(ctx->d_mats);
+  for (int i = 0; i < 7; ++i)
+    if (ctx->plan[i].d_vecs) cudaFree(ctx->plan[i].d_vecs);
+  if (ctx->d_err) cudaFree(ctx->d_err);
+  delete ctx;
+}
+
+int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_t stream) {
+  if (!ctx || !dst || !ctx->ws) return GNN_ERR_INVALID_ARG;
+  const int64_t N = ctx->last_nodes, E = ctx->last_edges, H = ctx->cfg.hidden;
+  const void* src = nullptr;
+  size_t need = 0;
+  switch (which) {
+    case 0: src = ctx->rowptr; need = 4 * (size_t)(N + 1); break;
+    case 1: src = ctx->perm; need = 4 * (size_t)E; break;
+    case 2: src = ctx->src_sorted; need = 4 * (size_t)E; break;
+    case 3: src = ctx->h; need = 4 * (size_t)(N * H); break;
+    case 4: src = ctx->e; need = 4 * (size_t)(E * H); break;
+    default: return GNN_ERR_INVALID_ARG;
+  }
+  if (bytes < need) return GNN_ERR_INVALID_ARG;
+  const cudaError_t err = cudaMemcpyAsync(dst, src, need, cudaMemcpyDeviceToDevice, (cudaStream_t)stream);
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
+
+}  // extern "C"

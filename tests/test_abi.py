@@ -1,0 +1,58 @@
+"""The C ABI library loads and exports every function include/gnn.h declares (no GPU calls)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "gnn.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(gnn_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ("gnn_create", "gnn_infer", "gnn_destroy", "gnn_status", "gnn_error_string"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    from paper_2402_09633_gb300 import build
+    path = build.build()
+    lib = ctypes.CDLL(path)
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_error_strings_without_gpu():
+    from paper_2402_09633_gb300 import binding
+    lib = binding.load_library()
+    assert lib.gnn_error_string(0) == b"ok"
+    assert lib.gnn_error_string(-5) == b"edge endpoint out of range"
+
+
+def test_invalid_arguments_rejected_on_host():
+    """Host-side validation returns codes before touching the device."""
+    from paper_2402_09633_gb300 import binding
+    lib = binding.load_library()
+    h = ctypes.c_void_p()
+    cfg = binding.GnnConfig(1, 3, 2, 96, 2, 2, 0, 1e-5)      # H = 96 unsupported
+    assert lib.gnn_create(ctypes.byref(cfg), ctypes.c_char_p(b"x" * 64), 64, ctypes.byref(h)) == -1
+    assert lib.gnn_create(None, None, 0, ctypes.byref(h)) == -1
+    assert lib.gnn_infer(None, None, None, 0, 0, None, None) == -1
+    assert lib.gnn_reserve(None, 1, 1) == -1
+
+
+def test_python_path_fails_loudly_without_library(tmp_path):
+    from paper_2402_09633_gb300 import binding
+    saved = binding._lib
+    binding._lib = None
+    try:
+        with pytest.raises(RuntimeError):
+            binding.load_library(str(tmp_path / "missing.so"))
+    finally:
+        binding._lib = saved
