@@ -1,0 +1,350 @@
+#!/usr/bin/env python
+"""Throughput of the interaction-network edge classifier on GB300.
+
+One step = one gnn_infer call on one synthetic full event (300,000 nodes,
+1,000,000 candidate edges, 12 node features, H=128, T=8, 3-layer MLPs):
+device-side CSR build, encoders, eight message-passing iterations and the
+classifier, inputs resident in HBM.  Prints one JSON line (rank 0).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+
+N > 1 runs under torchrun: every rank scores its own event (independent
+events, no data-path collective), so scaling is weak and `value` is the sum
+over ranks.  `--impl reference` times the fp64 CPU oracle on a bounded sample
+of the same workload (rank 0 only)."""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2402_09633_gb300 import synthetic as S  # noqa: E402
+
+METRIC = "GNN inference edges/sec and events/sec (300k-node/1M-edge) on 1 GB300; % of roofline"
+UNIT = "edges/s"
+L2_FLUSH_BYTES = 256 << 20          # > 2x the 129 MB L2, written between timed steps
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ------------------------------------------------------------------ traffic model
+def step_model(w: S.Workload):
+    """Algorithmic bytes and flops of one step (whole path) and of the two iteration kernels."""
+    m, ev = w.model, w.event
+    N, E = ev.n_nodes * w.n_events, ev.n_edges * w.n_events
+    H, T, L, Fn, s = m.hidden, m.n_iters, m.mlp_layers, m.n_node_feat, 4
+    bytes_step = (32 * E + 4 * N + 4 * Fn * N + (E + N) * H * s
+                  + T * ((3 * E + 2 * N) * H * s + 4 * E + 4 * N) + (2 * E + N) * H * s + 8 * E)
+    mac_edge_iter = E * H * H * L                           # e * W_e, then L-1 H x H layers
+    mac_node_iter = N * (2 * H * H + 2 * H * H + H * H * (L - 1))   # P_s, P_d, [h,a] layer, rest
+    flops_step = 2 * (T * (mac_edge_iter + mac_node_iter)
+                      + N * (Fn * H + H * H * (L - 1) + 2 * H * H)      # node encoder + projections
+                      + E * (2 * H + H * H * (L - 1))                   # edge encoder
+                      + E * (H * H * L + H))                            # classifier (+ head)
+    edge_update = {"bytes": E * (3 * H * s + 8) + N * H * s, "flops": 2 * mac_edge_iter,
+                   "bytes_note": "per edge: e read + e write + gathered W_s h_src row + 2 indices; "
+                                 "per node: W_d h_dst + b1 row"}
+    node_update = {"bytes": E * H * s + N * (5 * H * s + 8), "flops": 2 * mac_node_iter,
+                   "bytes_note": "per edge: message row of the CSR segment sum; per node: h read+write, "
+                                 "P_s/P_d write, its first-layer row, row pointers"}
+    return {"bytes": bytes_step, "flops": flops_step, "N": N, "E": E,
+            "edge_update": edge_update, "node_update": node_update}
+
+
+# ------------------------------------------------------------------ clocks
+def gpu_index_for(local_rank: int) -> str:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        items = [v.strip() for v in vis.split(",") if v.strip()]
+        if local_rank < len(items):
+            return items[local_rank]
+    return str(local_rank)
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: str):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", gpu, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, power, reasons = [], [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0])); smax.append(float(parts[1])); power.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ CPU oracle sample
+def oracle_sample(w: S.Workload, scale: float, seed: int = 0):
+    """A bounded sample of the workload: the same generator and model at `scale` of the event."""
+    ev = w.event
+    spec = S.EventSpec(max(int(ev.n_nodes * scale), 20), ev.n_extra_feat, ev.mode, ev.dphi_window,
+                       ev.fanout, max(int(ev.n_edges * scale), 1) if ev.mode == "powerlaw" else 0)
+    x, ei = S.generate_event(spec, seed)
+    W = S.init_weights(w.model, w.weight_seed)
+    return W, x, ei
+
+
+def time_oracle(w: S.Workload, scale: float, repeats: int = 1):
+    from oracle import gnn_oracle as O       # CPU baseline leg only
+    W, x, ei = oracle_sample(w, scale)
+    O.forward(W, x[:50], ei[:, :0], w.model.n_iters)          # import / allocator warm-up
+    times = []
+    for _ in range(repeats):
+        t0 = time.perf_counter()
+        O.forward(W, x, ei, w.model.n_iters, w.model.ln_eps)
+        times.append(time.perf_counter() - t0)
+    return ei.shape[1], x.shape[0], times
+
+
+def cpu_cores() -> int:
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    return os.cpu_count() or 1
+
+
+# ------------------------------------------------------------------ reference arm
+def run_reference(args, rank: int):
+    if rank != 0:
+        return
+    w = S.WORKLOADS[args.workload]
+    total = args.steps + args.warmup
+    scale = 0.01 if total <= 60 else 0.003
+    edges_per_step = []
+    times = []
+    for k in range(total):
+        e, n, t = time_oracle(w, scale, 1)
+        if k >= args.warmup:
+            times.append(t[0]); edges_per_step.append(e)
+    sec = sum(times)
+    value = sum(edges_per_step) / sec
+    sample = (f"{n} nodes / {e} edges from the '{w.name}' generator ({scale:g} of the event), "
+              f"same model (H={w.model.hidden}, T={w.model.n_iters}, L={w.model.mlp_layers}), fp64 numpy")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sec / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(w),
+            "events_per_s": value / w.event.n_edges,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def workload_config(w: S.Workload):
+    m, ev = w.model, w.event
+    return {"workload": w.name, "description": w.description, "n_nodes": ev.n_nodes * w.n_events,
+            "n_edges": ev.n_edges * w.n_events, "events_per_step": w.n_events,
+            "node_features": m.n_node_feat, "hidden": m.hidden, "n_iters": m.n_iters,
+            "mlp_layers": m.mlp_layers, "l2": "256 MB buffer written between timed steps",
+            "parallelism": "replicas (one event per GPU per step)"}
+
+
+# ------------------------------------------------------------------ GB300 arm
+def run_gb300(args, rank: int, world: int, local: int):
+    import torch
+    import torch.distributed as dist
+    from paper_2402_09633_gb300 import InteractionNetwork
+    from paper_2402_09633_gb300 import build as B
+
+    if rank == 0 or world == 1:
+        B.build()
+    if world > 1:
+        dist.init_process_group("nccl")
+        dist.barrier()
+        B.build()                       # no-op once rank 0 finished
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = S.WORKLOADS[args.workload]
+    x_np, ei_np = (S.generate_batch(w.event, [s + rank * w.n_events for s in w.seeds])
+                   if w.n_events > 1 else S.generate_event(w.event, w.seeds[0] + rank))
+    N, E = x_np.shape[0], ei_np.shape[1]
+    W = S.init_weights(w.model, w.weight_seed)
+    net = InteractionNetwork(w.model, S.pack_blob(w.model, W))
+    net.reserve(N, E)
+    x = torch.from_numpy(x_np).to(dev)
+    ei = torch.from_numpy(ei_np).to(dev)
+    scores = torch.empty(E, dtype=torch.float32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(args.warmup):
+        flush.fill_(1.0)
+        net.infer(x, ei, scores)
+    torch.cuda.synchronize(dev)
+    if net.status() != 0:
+        raise RuntimeError("device error during warm-up")
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(gpu_index_for(local))
+    time.sleep(0.3)
+    net.profile(True)
+    net.profile_read()                                   # clear
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t_wall = time.perf_counter()
+    for k in range(args.steps):
+        flush.fill_(float(k))
+        starts[k].record(stream)
+        net.infer(x, ei, scores)
+        ends[k].record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    wall = time.perf_counter() - t_wall
+    clocks = sampler.stop()
+    prof = net.profile_read()
+    net.profile(False)
+    status = net.status()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    mean_ms = sum(step_ms) / len(step_ms)
+    if world > 1:
+        t = torch.tensor([mean_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        mean_ms = float(t.item())
+    value = world * E / (mean_ms * 1e-3)
+
+    # end to end through the host-buffer entry point (copies inside the timed region)
+    x_h = torch.from_numpy(x_np).pin_memory()
+    ei_h = torch.from_numpy(ei_np).pin_memory()
+    s_h = torch.empty(E, dtype=torch.float32).pin_memory()
+    n_e2e = max(3, min(args.steps, 50))
+    net.infer_host(x_h, ei_h, s_h)
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(n_e2e):
+        net.infer_host(x_h, ei_h, s_h)
+    e2e_s = (time.perf_counter() - t0) / n_e2e
+    if world > 1:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e_ok = bool(np.array_equal(s_h.numpy(), scores.cpu().numpy()))
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    peaks, peak_src = load_peaks()
+    model = step_model(w)
+    groups = {g: {"ms_total": ms, "launches": n} for g, (ms, n) in prof.items() if n}
+    kernels_only = {g: v for g, v in groups.items() if g != "host_copies"}
+    dom = max(kernels_only, key=lambda g: kernels_only[g]["ms_total"])
+    dom_avg_s = kernels_only[dom]["ms_total"] * 1e-3 / kernels_only[dom]["launches"]
+    dom_model = model.get(dom, None)
+    roofline = None
+    if dom_model is not None:
+        achieved = dom_model["bytes"] / dom_avg_s / 1e9
+        roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"],
+                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                    "peak_source": f"{peak_src} (hbm_gbs, copy burst) -- of {peak_src}",
+                    "bytes_per_launch": dom_model["bytes"], "avg_launch_ms": dom_avg_s * 1e3,
+                    "tensor_tflops_executed": 3 * dom_model["flops"] / dom_avg_s / 1e12}
+    t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9),
+                          model["flops"] / (peaks["bf16_tflops"] * 1e12))
+    total_launches = sum(v["launches"] for v in kernels_only.values())
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        scale = 0.1
+        e_s, n_s, t = time_oracle(w, scale, 1)
+        cpu = {"value": e_s / t[0], "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{n_s} nodes / {e_s} edges from the '{w.name}' generator ({scale:g} of the "
+                         f"event), same model, fp64 numpy, one pass of {t[0]:.1f} s"}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": mean_ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16x3->f32", "data": "synthetic",
+            "config": workload_config(w),
+            "events_per_s": value / E * w.n_events,
+            "roofline": roofline,
+            "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms,
+                              "bytes_alg": model["bytes"], "flops_alg": model["flops"]},
+            "kernels": groups,
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * E / e2e_s, "unit": UNIT,
+                    "h2d_bytes_per_step": int(x_np.nbytes + ei_np.nbytes),
+                    "d2h_bytes_per_step": int(E * 4), "ms_per_step": e2e_s * 1e3,
+                    "matches_device_path": e2e_ok},
+            "gpu_launches": int(total_launches),
+            "clocks": clocks,
+            "device_status": status,
+            "wall_s_timed_region": wall}
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("gb300", "reference"), default="gb300")
+    ap.add_argument("--workload", choices=tuple(S.WORKLOADS), default="full")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local = int(os.environ.get("LOCAL_RANK", 0))
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args, rank)
+    else:
+        run_gb300(args, rank, world, local)
+
+
+if __name__ == "__main__":
+    main()

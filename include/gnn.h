@@ -118,6 +118,35 @@ int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, 
               int64_t n_edges, float* edge_scores, gnn_stream_t stream);
 
 /*
+ * gnn_infer_host -- gnn_infer on HOST buffers (the form a serving backend
+ * receives requests in): copies node_feats [n_nodes, n_node_feat] float32 and
+ * edge_index [2, n_edges] int32 from host memory into the context's staging
+ * buffers, scores on the device, copies the scores back into edge_scores
+ * [n_edges] float32 (host), and synchronises `stream` before returning.
+ * Pinned (page-locked) host memory makes the copies asynchronous DMA;
+ * pageable memory also works.  Same argument rules and errors as gnn_infer,
+ * plus the device status of this call (as gnn_status would return it).
+ */
+int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
+                   int64_t n_edges, float* edge_scores, gnn_stream_t stream);
+
+/*
+ * gnn_profile_enable -- when on != 0, later gnn_infer / gnn_infer_host calls
+ * record a CUDA event pair on their stream around every kernel group, so
+ * gnn_profile_read can report device time per group.  Off by default.
+ *
+ * gnn_profile_read -- synchronise the recorded events and write, for each
+ * group g < n_groups, the summed device milliseconds ms[g] and the number of
+ * kernel launches launches[g]; then clear the records.  Groups: 0 CSR build
+ * (all its kernels), 1 node encoder, 2 edge encoder, 3 edge update, 4 node
+ * update, 5 classifier, 6 host<->device copies of gnn_infer_host, 7 message
+ * aggregation.  Either output pointer may be NULL.  Returns the number of
+ * groups (8) or an error.
+ */
+int gnn_profile_enable(gnn_ctx* ctx, int on);
+int gnn_profile_read(gnn_ctx* ctx, double* ms, int64_t* launches, int n_groups);
+
+/*
  * gnn_status -- synchronise `stream`, then return and clear the device error
  * word of the context: GNN_OK, GNN_ERR_INDEX_RANGE, GNN_ERR_DEVICE_TIMEOUT or
  * GNN_ERR_CUDA (a failed synchronisation).
@@ -134,9 +163,11 @@ const char* gnn_error_string(int code);
  * gnn_debug_copy -- test hook: copy an internal buffer of the last gnn_infer
  * into caller device memory `dst` of at least `bytes` bytes (enqueued on
  * `stream`).  which: 0 rowptr int32 [N+1], 1 perm int32 [E] (CSR slot ->
- * input edge id), 2 src_sorted int32 [E], 3 node state h float32 [N, H],
- * 4 edge state e float32 [E, H] in CSR order.  Errors: INVALID_ARG when the
- * buffer is unknown or `bytes` is too small.
+ * input edge id), 2 src_sorted int32 [E], 3 node state h, 4 edge state e (CSR
+ * order).  The states are float32 in the row-tiled layout of the kernels:
+ * R = rows rounded up to a multiple of 128, element (r, c) at index
+ * ((r / 128) * (H / 8) + c / 8) * 1024 + (r % 128) * 8 + c % 8, R * H floats.
+ * Errors: INVALID_ARG when the buffer is unknown or `bytes` is too small.
  */
 int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_t stream);
 

@@ -14,8 +14,11 @@ _lib = None
 GNN_OK = 0
 ERRORS = {-1: "INVALID_ARG", -2: "BAD_WEIGHTS", -3: "OOM", -4: "CUDA", -5: "INDEX_RANGE",
           -6: "DEVICE_TIMEOUT"}
-EXPORTED = ("gnn_create", "gnn_reserve", "gnn_infer", "gnn_status", "gnn_destroy",
-            "gnn_error_string", "gnn_debug_copy")
+EXPORTED = ("gnn_create", "gnn_reserve", "gnn_infer", "gnn_infer_host", "gnn_status",
+            "gnn_destroy", "gnn_error_string", "gnn_debug_copy", "gnn_profile_enable",
+            "gnn_profile_read")
+PROFILE_GROUPS = ("csr_build", "node_encoder", "edge_encoder", "edge_update", "node_update",
+                  "classifier", "host_copies", "aggregate")
 
 
 class GnnError(RuntimeError):
@@ -54,6 +57,12 @@ def load_library(path: str = LIB_PATH):
     lib.gnn_error_string.restype = ctypes.c_char_p
     lib.gnn_debug_copy.argtypes = [vp, i32, vp, ctypes.c_size_t, vp]
     lib.gnn_debug_copy.restype = i32
+    lib.gnn_infer_host.argtypes = [vp, vp, vp, i64, i64, vp, vp]
+    lib.gnn_infer_host.restype = i32
+    lib.gnn_profile_enable.argtypes = [vp, i32]
+    lib.gnn_profile_enable.restype = i32
+    lib.gnn_profile_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64), i32]
+    lib.gnn_profile_read.restype = i32
     _lib = lib
     return lib
 
@@ -99,6 +108,34 @@ class InteractionNetwork:
         if rc != GNN_OK:
             raise GnnError(rc, "gnn_infer")
         return scores
+
+    def infer_host(self, x, edge_index, scores, stream=None) -> int:
+        """Host buffers in and out (numpy arrays or pinned CPU tensors); returns the status code."""
+        import numpy as np
+
+        def ptr(a):
+            return ctypes.c_void_p(a.data_ptr() if hasattr(a, "data_ptr") else a.ctypes.data)
+        n, e = x.shape[0], edge_index.shape[1]
+        if isinstance(x, np.ndarray):
+            assert x.dtype == np.float32 and edge_index.dtype == np.int32 and scores.dtype == np.float32
+            assert x.flags.c_contiguous and edge_index.flags.c_contiguous
+        rc = self.lib.gnn_infer_host(self.handle, ptr(x), ptr(edge_index), n, e, ptr(scores),
+                                     _stream_handle(stream))
+        if rc not in (GNN_OK, -5):
+            raise GnnError(rc, "gnn_infer_host")
+        return rc
+
+    def profile(self, on: bool = True):
+        self.lib.gnn_profile_enable(self.handle, 1 if on else 0)
+
+    def profile_read(self) -> dict:
+        n = len(PROFILE_GROUPS)
+        ms = (ctypes.c_double * n)()
+        cnt = (ctypes.c_int64 * n)()
+        rc = self.lib.gnn_profile_read(self.handle, ms, cnt, n)
+        if rc < 0:
+            raise GnnError(rc, "gnn_profile_read")
+        return {g: (ms[i], cnt[i]) for i, g in enumerate(PROFILE_GROUPS)}
 
     def status(self, stream=None) -> int:
         return self.lib.gnn_status(self.handle, _stream_handle(stream))

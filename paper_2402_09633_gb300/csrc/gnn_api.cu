@@ -61,8 +61,20 @@ struct gnn_ctx {
   int *keys_a = nullptr, *keys_b = nullptr, *vals_a = nullptr, *vals_b = nullptr, *src_c = nullptr;
   int *hist = nullptr, *perm = nullptr, *src_sorted = nullptr, *dst_sorted = nullptr, *rowptr = nullptr;
   int* key_sorted = nullptr;
-  float *e = nullptr, *h = nullptr, *ps = nullptr, *pd = nullptr;
+  float *e = nullptr, *h = nullptr, *ps = nullptr, *pd = nullptr, *agg = nullptr;
   int64_t last_nodes = 0, last_edges = 0;
+  // staging for gnn_infer_host
+  void* stage = nullptr;
+  size_t stage_bytes = 0;
+  // profiling: event pairs around kernel groups
+  struct ProfRec { int group; int launches; cudaEvent_t a, b; };
+  bool prof_on = false;
+  std::vector<ProfRec> prof;
+  size_t prof_used = 0;
+#ifdef GNN_TRACE
+  unsigned long long* trace = nullptr;   // stamps of CTA 0 of the traced kernel kind
+  int trace_kind = -1;
+#endif
 };
 
 namespace {
@@ -111,6 +123,26 @@ int cuda_fail(cudaError_t e) {
   return e == cudaErrorMemoryAllocation ? GNN_ERR_OOM : GNN_ERR_CUDA;
 }
 
+constexpr int kProfGroups = 8;
+
+// Returns the record index, or -1 when profiling is off.
+int prof_begin(gnn_ctx* c, int group, int launches, cudaStream_t st) {
+  if (!c->prof_on) return -1;
+  if (c->prof_used == c->prof.size()) {
+    gnn_ctx::ProfRec r{};
+    if (cudaEventCreate(&r.a) != cudaSuccess || cudaEventCreate(&r.b) != cudaSuccess) return -1;
+    c->prof.push_back(r);
+  }
+  gnn_ctx::ProfRec& r = c->prof[c->prof_used];
+  r.group = group;
+  r.launches = launches;
+  cudaEventRecord(r.a, st);
+  return (int)c->prof_used++;
+}
+void prof_end(gnn_ctx* c, int idx, cudaStream_t st) {
+  if (idx >= 0) cudaEventRecord(c->prof[idx].b, st);
+}
+
 template <TileKind K, int H>
 cudaError_t set_smem_attr() {
   return cudaFuncSetAttribute(mlp_tile_kernel<K, H>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -128,7 +160,7 @@ cudaError_t set_all_attrs() {
 }
 
 template <TileKind K, int H>
-void launch_tile(const gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st) {
+void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st) {
   p.n_jobs = pl.n_jobs;
   for (int j = 0; j < kMaxJobs; ++j) { p.job_mat[j] = pl.job_mat[j]; p.job_acc[j] = pl.job_acc[j]; }
   p.vecs = pl.d_vecs;
@@ -141,7 +173,13 @@ void launch_tile(const gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStrea
   if (smem < 120 * 1024) smem = 120 * 1024;           // one CTA per SM (it owns the TMEM)
   const int pairs = (p.n_tiles + 1) / 2;
   const int grid = pairs < c->n_sm ? pairs : c->n_sm;
+#ifdef GNN_TRACE
+  p.trace = ((int)K == c->trace_kind) ? c->trace : nullptr;
+#endif
+  static const int group[5] = {1, 2, 3, 4, 5};      // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier
+  const int pr = prof_begin(c, group[(int)K], 1, st);
   mlp_tile_kernel<K, H><<<grid, kThreads, smem, st>>>(p);
+  prof_end(c, pr, st);
 }
 
 template <int H>
@@ -157,7 +195,7 @@ int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStr
   p.key_sorted = c->key_sorted;
   p.perm = c->perm;
   p.rowptr = c->rowptr;
-  p.e = c->e; p.h = c->h; p.ps = c->ps; p.pd = c->pd;
+  p.e = c->e; p.h = c->h; p.ps = c->ps; p.pd = c->pd; p.agg = c->agg;
   p.scores = scores;
   p.err = c->d_err;
   const int T = c->cfg.n_iters;
@@ -168,6 +206,12 @@ int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStr
   launch_tile<TileKind::EdgeEncoder, H>(c, c->plan[2], pe, st);
   for (int t = 1; t <= T; ++t) {
     launch_tile<TileKind::EdgeUpdate, H>(c, c->plan[3], pe, st);
+    {
+      const int pr = prof_begin(c, 7, 1, st);
+      const dim3 grid((N + 31) / 32, (H / 8 + 7) / 8);
+      aggregate_kernel<H><<<grid, 256, 0, st>>>(c->e, c->rowptr, N, c->agg);
+      prof_end(c, pr, st);
+    }
     launch_tile<TileKind::NodeUpdate, H>(c, c->plan[t < T ? 4 : 5], pn, st);
   }
   launch_tile<TileKind::Classifier, H>(c, c->plan[6], pe, st);
@@ -189,8 +233,11 @@ int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
   const int64_t rs_tiles = (e + kRadixTile - 1) / kRadixTile;
   auto al = [](int64_t b) { return (b + 255) & ~int64_t(255); };
   const int64_t sz_e_int = al(4 * (e > 0 ? e : 1));
+  // edge and node state use the row-tiled layout: rows padded to whole 128-row tiles
+  const int64_t e_pad = (e + kTileRows - 1) / kTileRows * kTileRows;
+  const int64_t n_pad = (n + kTileRows - 1) / kTileRows * kTileRows;
   const int64_t total = 8 * sz_e_int + al(4 * 256 * (rs_tiles > 0 ? rs_tiles : 1)) + al(4 * (n + 1)) +
-                        al(4 * e * H) + 3 * al(4 * n * H);
+                        al(4 * e_pad * H) + 2 * al(4 * n_pad * H) + 2 * al(4 * n * H);
   free_workspace(c);
   void* ws = nullptr;
   cudaError_t err = cudaMalloc(&ws, (size_t)total);
@@ -204,8 +251,9 @@ int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
   c->src_sorted = (int*)take(4 * e); c->dst_sorted = (int*)take(4 * e);
   c->hist = (int*)take(4 * 256 * (rs_tiles > 0 ? rs_tiles : 1));
   c->rowptr = (int*)take(4 * (n + 1));
-  c->e = (float*)take(4 * e * H);
-  c->h = (float*)take(4 * n * H);
+  c->e = (float*)take(4 * e_pad * H);
+  c->h = (float*)take(4 * n_pad * H);
+  c->agg = (float*)take(4 * n_pad * H);
   c->ps = (float*)take(4 * n * H);
   c->pd = (float*)take(4 * n * H);
   c->cap_nodes = n;
@@ -215,6 +263,10 @@ int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
 
 int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
   const int tb = 256;
+  int n_bits = 0;
+  while (n_bits < 31 && (N >> n_bits) != 0) ++n_bits;
+  const int n_passes = ((n_bits > 0 ? n_bits : 1) + 7) / 8;
+  const int pr = prof_begin(c, 0, 3 + 3 * n_passes, st);
   csr_keys_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(ei, E, N, c->keys_a, c->vals_a, c->src_c, c->d_err);
   int bits = 0;
   while (bits < 31 && (N >> bits) != 0) ++bits;        // keys lie in [0, N]
@@ -234,6 +286,7 @@ int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
   csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, c->src_c, E, N, c->perm, c->src_sorted,
                                                      c->dst_sorted);
   csr_rowptr_kernel<<<(E + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, c->rowptr);
+  prof_end(c, pr, st);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
@@ -332,7 +385,8 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     add_deep(pl, NODE_ENC);
     pl.job_mat[pl.n_jobs++] = target == 0 ? en_s : cl_s;
     pl.job_mat[pl.n_jobs++] = target == 0 ? en_d : cl_d;
-    push(pl.vecs, lay[NODE_ENC][0].W, (size_t)H * Fn);
+    for (int k = 0; k < Fn; ++k)                        // first-layer weight, transposed
+      for (int i = 0; i < H; ++i) pl.vecs.push_back(lay[NODE_ENC][0].W[(size_t)i * Fn + k]);
     bgb(pl.vecs, NODE_ENC, 0);
     push(pl.vecs, lay[target == 0 ? EDGE_NET : CLASSIFIER][0].b, H);
   }
@@ -340,7 +394,8 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     KernelPlan& pl = c->plan[2];
     pl.n_jobs = 0;
     add_deep(pl, EDGE_ENC);
-    push(pl.vecs, lay[EDGE_ENC][0].W, (size_t)H * 2);
+    for (int k = 0; k < 2; ++k)
+      for (int i = 0; i < H; ++i) pl.vecs.push_back(lay[EDGE_ENC][0].W[(size_t)i * 2 + k]);
     bgb(pl.vecs, EDGE_ENC, 0);
   }
   {  // edge update
@@ -379,6 +434,11 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     if (err == cudaSuccess)
       err = cudaMemcpy(c->plan[i].d_vecs, c->plan[i].vecs.data(), c->plan[i].vecs.size() * 4, cudaMemcpyHostToDevice);
   }
+#ifdef GNN_TRACE
+  if (err == cudaSuccess) err = cudaMalloc(&c->trace, 3 * kTraceEvents * 8);
+  if (err == cudaSuccess) err = cudaMemset(c->trace, 0, 3 * kTraceEvents * 8);
+  if (const char* k = getenv("GNN_TRACE_KIND")) c->trace_kind = atoi(k);
+#endif
   if (err == cudaSuccess) err = cudaMalloc(&c->d_err, 4);
   if (err == cudaSuccess) err = cudaMemset(c->d_err, 0, 4);
   if (err != cudaSuccess) { gnn_destroy(c); return cuda_fail(err); }
@@ -410,6 +470,74 @@ int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, 
                                 : run_network<64>(ctx, node_feats, N, E, edge_scores, st);
 }
 
+int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
+                   int64_t n_edges, float* edge_scores, gnn_stream_t stream) {
+  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX)
+    return GNN_ERR_INVALID_ARG;
+  if (n_edges == 0) return GNN_OK;
+  if (n_nodes == 0 || !node_feats || !edge_index || !edge_scores) return GNN_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  const size_t bx = (size_t)n_nodes * ctx->cfg.n_node_feat * 4, be = (size_t)n_edges * 8,
+               bs = (size_t)n_edges * 4;
+  auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+  const size_t need = al(bx) + al(be) + al(bs);
+  if (need > ctx->stage_bytes) {
+    if (ctx->stage) { cudaStreamSynchronize(st); cudaFree(ctx->stage); ctx->stage = nullptr; ctx->stage_bytes = 0; }
+    const cudaError_t err = cudaMalloc(&ctx->stage, need);
+    if (err != cudaSuccess) return cuda_fail(err);
+    ctx->stage_bytes = need;
+  }
+  uint8_t* q = (uint8_t*)ctx->stage;
+  float* dx = (float*)q;
+  int32_t* de = (int32_t*)(q + al(bx));
+  float* ds = (float*)(q + al(bx) + al(be));
+  int pr = prof_begin(ctx, 6, 2, st);
+  cudaError_t err = cudaMemcpyAsync(dx, node_feats, bx, cudaMemcpyHostToDevice, st);
+  if (err == cudaSuccess) err = cudaMemcpyAsync(de, edge_index, be, cudaMemcpyHostToDevice, st);
+  prof_end(ctx, pr, st);
+  if (err != cudaSuccess) return cuda_fail(err);
+  int rc = gnn_infer(ctx, dx, de, n_nodes, n_edges, ds, stream);
+  if (rc != GNN_OK) return rc;
+  pr = prof_begin(ctx, 6, 1, st);
+  err = cudaMemcpyAsync(edge_scores, ds, bs, cudaMemcpyDeviceToHost, st);
+  prof_end(ctx, pr, st);
+  if (err != cudaSuccess) return cuda_fail(err);
+  return gnn_status(ctx, stream);
+}
+
+#ifdef GNN_TRACE
+int gnn_trace_read(gnn_ctx* ctx, unsigned long long* host) {
+  cudaDeviceSynchronize();
+  return cudaMemcpy(host, ctx->trace, 3 * kTraceEvents * 8, cudaMemcpyDeviceToHost) == cudaSuccess ? 0 : -4;
+}
+#endif
+
+int gnn_profile_enable(gnn_ctx* ctx, int on) {
+  if (!ctx) return GNN_ERR_INVALID_ARG;
+  ctx->prof_on = on != 0;
+  return GNN_OK;
+}
+
+int gnn_profile_read(gnn_ctx* ctx, double* ms, int64_t* launches, int n_groups) {
+  if (!ctx || n_groups < 0) return GNN_ERR_INVALID_ARG;
+  double acc[kProfGroups] = {0};
+  int64_t cnt[kProfGroups] = {0};
+  for (size_t i = 0; i < ctx->prof_used; ++i) {
+    gnn_ctx::ProfRec& r = ctx->prof[i];
+    if (cudaEventSynchronize(r.b) != cudaSuccess) return cuda_fail(cudaGetLastError());
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) return cuda_fail(cudaGetLastError());
+    acc[r.group] += t;
+    cnt[r.group] += r.launches;
+  }
+  ctx->prof_used = 0;
+  for (int g = 0; g < n_groups && g < kProfGroups; ++g) {
+    if (ms) ms[g] = acc[g];
+    if (launches) launches[g] = cnt[g];
+  }
+  return kProfGroups;
+}
+
 int gnn_status(gnn_ctx* ctx, gnn_stream_t stream) {
   if (!ctx) return GNN_ERR_INVALID_ARG;
   cudaError_t err = cudaStreamSynchronize((cudaStream_t)stream);
@@ -431,6 +559,8 @@ void gnn_destroy(gnn_ctx* ctx) {
   for (int i = 0; i < 7; ++i)
     if (ctx->plan[i].d_vecs) cudaFree(ctx->plan[i].d_vecs);
   if (ctx->d_err) cudaFree(ctx->d_err);
+  if (ctx->stage) cudaFree(ctx->stage);
+  for (auto& r : ctx->prof) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }
   delete ctx;
 }
 
@@ -443,8 +573,8 @@ int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_
     case 0: src = ctx->rowptr; need = 4 * (size_t)(N + 1); break;
     case 1: src = ctx->perm; need = 4 * (size_t)E; break;
     case 2: src = ctx->src_sorted; need = 4 * (size_t)E; break;
-    case 3: src = ctx->h; need = 4 * (size_t)(N * H); break;
-    case 4: src = ctx->e; need = 4 * (size_t)(E * H); break;
+    case 3: src = ctx->h; need = 4 * (size_t)((N + kTileRows - 1) / kTileRows * kTileRows * H); break;
+    case 4: src = ctx->e; need = 4 * (size_t)((E + kTileRows - 1) / kTileRows * kTileRows * H); break;
     default: return GNN_ERR_INVALID_ARG;
   }
   if (bytes < need) return GNN_ERR_INVALID_ARG;

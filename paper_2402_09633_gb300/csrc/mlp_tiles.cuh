@@ -14,12 +14,12 @@
 // Roles (576 threads = 18 warps):
 //   warp 0      : MMA issuer (one elected lane)
 //   warp 1      : weight producer (bulk copies into the smem weight ring)
-//   warps 2..17 : 16 row-worker warps = 2 slots x 2 column halves x 4 lane
-//                 quarters.  Slot s works on tiles 2p+s of tile pair p, so the
-//                 tensor core alternates between the two slots (ping-pong) and
-//                 one slot's epilogue overlaps the other slot's MMAs.
-// Each row of a tile is owned by two threads (column halves); LayerNorm
-// statistics are combined through a small shared-memory exchange.
+//   warps 2..17 : 16 row-worker warps, 8 per slot.  Slot s works on tile
+//                 2p+s of tile pair p; the issuer serves whichever slot is
+//                 ready, so one slot's epilogue overlaps the other slot's MMAs.
+// A worker warp owns 16 rows of a tile; a quad of threads shares two rows
+// (each thread a quarter of the columns), reads them from tensor memory with
+// the 16-lane shapes and does LayerNorm / ReLU in registers.
 #pragma once
 #include <cstdint>
 #include <cuda_bf16.h>
@@ -65,9 +65,28 @@ struct TileParams {
   float* h;                   // [N, H] node state
   float* ps;                  // [N, H] projections W_s h
   float* pd;                  // [N, H] projections W_d h + b1
+  float* agg;                 // [N, H] row-tiled: sum of incoming messages per node
   float* scores;              // [E] input order
   uint32_t* err;              // device error word
+#ifdef GNN_TRACE
+  unsigned long long* trace;  // [3 roles][kTraceEvents] %globaltimer stamps of CTA 0
+#endif
 };
+
+#ifdef GNN_TRACE
+constexpr int kTraceEvents = 512;
+#define GNN_TRACE_AT(role, idx)                                                               \
+  do {                                                                                        \
+    if (p.trace && blockIdx.x == 0 && (idx) < kTraceEvents) p.trace[(role) * kTraceEvents + (idx)] = global_timer_ns(); \
+  } while (0)
+#define GNN_TRACE_W(label)                                                                   \
+  do {                                                                                       \
+    if (slot == 0 && trow == 0) GNN_TRACE_AT(1, tr_iter * 16 + (label));                     \
+  } while (0)
+#else
+#define GNN_TRACE_AT(role, idx) do { } while (0)
+#define GNN_TRACE_W(label) do { } while (0)
+#endif
 
 template <int H>
 struct TileGeom {
@@ -87,27 +106,25 @@ __host__ __device__ constexpr int padded_vec_floats(int n) { return (n + 3) & ~3
 template <int H>
 constexpr uint32_t tile_smem_bytes(int n_vec_floats) {
   // ring (1024-aligned) + vectors + exchange buffers + barriers + alignment slack
-  return TileGeom<H>::RING_BYTES + (uint32_t)padded_vec_floats(n_vec_floats) * 4u + 2 * 2 * 2 * 128 * 4 +
-         256 + 1024;
+  return TileGeom<H>::RING_BYTES + (uint32_t)padded_vec_floats(n_vec_floats) * 4u + 256 + 1024;
 }
 
 // ----------------------------------------------------------------- kernel
 template <TileKind KIND, int H>
 __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams p) {
   using G = TileGeom<H>;
-  constexpr int HH = G::HH;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* ring = smem;
   float* vecs = reinterpret_cast<float*>(smem + G::RING_BYTES);
-  float* red = vecs + padded_vec_floats(p.n_vec_floats);    // [2 slot][2 buf][2 half][128]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(red + 2 * 2 * 2 * 128);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + padded_vec_floats(p.n_vec_floats));
   uint64_t* a_full = bars;          // [2]
   uint64_t* d_full = bars + 2;      // [2]
   uint64_t* w_full = bars + 4;      // [STAGES]
   uint64_t* w_empty = bars + 4 + G::STAGES;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * G::STAGES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* progress = abort_flag + 1;          // tile pair slot 0's workers are on (L2 prefetch pacing)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -117,8 +134,9 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
   if (threadIdx.x == 0) {
     mbar_init(&a_full[0], 8); mbar_init(&a_full[1], 8);
     mbar_init(&d_full[0], 1); mbar_init(&d_full[1], 1);
-    for (int s = 0; s < G::STAGES; ++s) { mbar_init(&w_full[s], 1); mbar_init(&w_empty[s], 1); }
+    for (int s = 0; s < G::STAGES; ++s) { mbar_init(&w_full[s], 1); mbar_init(&w_empty[s], 2); }
     *abort_flag = 0;
+    progress[0] = -1;
     fence_mbar_init();
   }
   if (warp == 0) { tmem_alloc(tmem_slot, G::TMEM_COLS); tmem_relinquish(); }
@@ -137,7 +155,36 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         mbar_arrive_expect_tx(&w_full[0], total);
         for (int j = 0; j < p.n_jobs; ++j)
           bulk_g2s(ring + j * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[0]);
-      } else {
+      }
+    }
+    __syncwarp();
+    if (resident && (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier)) {
+      // L2 prefetcher: while the workers are on tile pair k, warm L2 with the
+      // edge-state tiles and the gathered P_s / P_d rows of pair k+1.
+      const uint64_t t0 = global_timer_ns();
+      for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
+        const int prev = pair - (int)gridDim.x;
+        for (uint32_t it = 0; prev >= 0 && progress[0] < prev; ++it) {    // bounded: gives up silently
+          if (*abort_flag || ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs)) break;
+          __nanosleep(200);
+        }
+        for (int s = 0; s < 2; ++s) {
+          const int tile = 2 * pair + s;
+          if (tile >= p.n_tiles) break;
+          if (lane == 0) prefetch_l2_bulk(p.e + (size_t)tile * kTileRows * H, kTileRows * H * 4);
+#pragma unroll
+          for (int i = 0; i < kTileRows / 32; ++i) {
+            const int row = tile * kTileRows + i * 32 + lane;
+            if (row < p.n_rows) {
+              prefetch_l2_bulk(p.ps + (size_t)p.src_sorted[row] * H, H * 4);
+              prefetch_l2_bulk(p.pd + (size_t)p.dst_sorted[row] * H, H * 4);
+            }
+          }
+        }
+      }
+    }
+    if (!resident && lane == 0) {
+      {
         uint32_t seq = 0;
         for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
           for (int j = 0; j < p.n_jobs; ++j, ++seq) {
@@ -153,144 +200,209 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     __syncwarp();
   } else if (warp == 0) {
     // ------------------------------------------------ MMA issuer
+    // The two slots advance independently: each has its own job cursor, and
+    // the issuer serves whichever slot has published its next A operand.  In
+    // streamed-weight mode both slots walk the same (pair, job) sequence of
+    // ring stages; a stage is released after both slots' MMAs on it completed
+    // (w_empty counts two commits; a slot without a tile in the last pair is
+    // covered by a second commit of the other slot).
     if (lane == 0) {
-      uint32_t a_use[2] = {0, 0};
-      uint32_t seq = 0;
+      int pair_s[2] = {(int)blockIdx.x, (int)blockIdx.x};
+      int job_s[2] = {0, 0};
+      uint32_t seq_s[2] = {0, 0};
+      uint32_t a_par[2] = {0, 0};
+      bool act[2] = {2 * (int)blockIdx.x < p.n_tiles, 2 * (int)blockIdx.x + 1 < p.n_tiles};
       bool ok = true;
       if (resident) ok = bounded_wait(&w_full[0], 0, abort_flag, p.err);
-      for (int pair = blockIdx.x; ok && pair < n_pairs; pair += gridDim.x) {
-        const bool has1 = (2 * pair + 1) < p.n_tiles;
-        for (int j = 0; j < p.n_jobs && ok; ++j, ++seq) {
-          const int st = resident ? j : (int)(seq % G::STAGES);
-          if (!resident) ok = bounded_wait(&w_full[st], (seq / G::STAGES) & 1, abort_flag, p.err);
-          if (!ok) break;
-          const uint32_t wb = smem_u32(ring + st * G::MAT_BYTES);
-          for (int s = 0; s < 2 && ok; ++s) {
-            if (s == 1 && !has1) break;
-            ok = bounded_wait(&a_full[s], a_use[s] & 1, abort_flag, p.err);
-            a_use[s]++;
-            if (!ok) break;
-            tc_fence_after();
-            const uint32_t d = tmem_base + s * G::SLOT_COLS;
-            const uint32_t ahi = d + H, alo = d + H + H / 2;
+      uint64_t t_last = global_timer_ns();
+      uint32_t spins = 0;
+      while (ok && (act[0] || act[1])) {
+        bool progressed = false;
 #pragma unroll
-            for (int ks = 0; ks < H / 16; ++ks) {
-              const uint32_t off = (ks >> 2) * (H * 128) + (ks & 3) * 32;
-              const uint64_t bh = sdesc_kmajor_sw128(wb + off);
-              const uint64_t bl = sdesc_kmajor_sw128(wb + G::PART_BYTES + off);
-              const uint32_t acc = (p.job_acc[j] || ks > 0) ? 1u : 0u;
-              mma_bf16_ts(d, ahi + ks * 8, bh, G::IDESC, acc);
-              mma_bf16_ts(d, ahi + ks * 8, bl, G::IDESC, 1u);
-              mma_bf16_ts(d, alo + ks * 8, bh, G::IDESC, 1u);
-            }
-            mma_commit(&d_full[s]);
+        for (int s = 0; s < 2; ++s) {
+          if (!act[s]) continue;
+          const int j = job_s[s];
+          const int st = resident ? j : (int)(seq_s[s] % G::STAGES);
+          if (!resident && !mbar_test_wait(&w_full[st], (seq_s[s] / G::STAGES) & 1)) continue;
+          if (!mbar_test_wait(&a_full[s], a_par[s])) continue;
+          a_par[s] ^= 1;
+          GNN_TRACE_AT(0, 2 * (seq_s[0] + seq_s[1]));
+          tc_fence_after();
+          const uint32_t wb = smem_u32(ring + st * G::MAT_BYTES);
+          const uint32_t d = tmem_base + s * G::SLOT_COLS;
+          const uint32_t ahi = d + H, alo = d + H + H / 2;
+#pragma unroll
+          for (int ks = 0; ks < H / 16; ++ks) {
+            const uint32_t off = (ks >> 2) * (H * 128) + (ks & 3) * 32;
+            const uint64_t bh = sdesc_kmajor_sw128(wb + off);
+            const uint64_t bl = sdesc_kmajor_sw128(wb + G::PART_BYTES + off);
+            const uint32_t acc = (p.job_acc[j] || ks > 0) ? 1u : 0u;
+            mma_bf16_ts(d, ahi + ks * 8, bh, G::IDESC, acc);
+            mma_bf16_ts(d, ahi + ks * 8, bl, G::IDESC, 1u);
+            mma_bf16_ts(d, alo + ks * 8, bh, G::IDESC, 1u);
           }
-          if (!resident && ok) mma_commit(&w_empty[st]);
+          mma_commit(&d_full[s]);
+          GNN_TRACE_AT(0, 2 * (seq_s[0] + seq_s[1]) + 1);
+          if (!resident) {
+            mma_commit(&w_empty[st]);
+            if (s == 0 && 2 * pair_s[0] + 1 >= p.n_tiles) mma_commit(&w_empty[st]);   // slot 1 has no tile
+          }
+          seq_s[s]++;
+          if (++job_s[s] == p.n_jobs) {
+            job_s[s] = 0;
+            pair_s[s] += gridDim.x;
+            act[s] = 2 * pair_s[s] + s < p.n_tiles;
+          }
+          progressed = true;
+        }
+        if (progressed) {
+          t_last = global_timer_ns();
+          spins = 0;
+        } else if ((++spins & 63u) == 0) {
+          if (*abort_flag) break;
+          if (global_timer_ns() - t_last > kWaitLimitNs) {
+            atomicOr(p.err, DEV_ERR_TIMEOUT);
+            *abort_flag = 1;
+            break;
+          }
         }
       }
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------ row workers
-    const int wi = warp - 2;                 // 0..15
-    const int slot = wi >> 3;
-    const int half = (wi >> 2) & 1;
+    // ------------------------------------------------ row workers (quad layout)
+    // Worker warp w serves slot (w-2)/8 and the 16 TMEM lanes
+    // [32*(w%4) + 16*hq, +16) of its lane quarter (hq = ((w-2)/4) % 2).
+    // Thread t of the warp owns rows r0 = base + t/4 and r1 = r0 + 8 and, in
+    // every 8-column block b, columns 8b + 2(t%4) and 8b + 2(t%4) + 1: the four
+    // threads of a quad share two rows, so LayerNorm statistics reduce with
+    // two quad shuffles.  v[4b + {0,1}] = row r0, v[4b + {2,3}] = row r1.
+    constexpr int NB = H / 8;                // 8-column blocks per row
+    const int wq = warp - 2;                 // 0..15
+    const int slot = wq >> 3;
+    const int hq = (wq >> 2) & 1;
     const int quarter = warp & 3;            // TMEM lane quarter of this warp
-    const int trow = quarter * 32 + lane;    // row inside the tile
-    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    const uint32_t d_addr = tmem_base + slot * G::SLOT_COLS + lane_off + half * HH;
-    const uint32_t ahi_addr = tmem_base + slot * G::SLOT_COLS + H + lane_off + half * (HH / 2);
-    const uint32_t alo_addr = ahi_addr + H / 2;
-    float* red_slot = red + slot * (2 * 2 * 128);
-    uint32_t d_use = 0, xbuf = 0;
-    const int c0 = half * HH;                // first column of this thread
+    const int lane_base = quarter * 32 + hq * 16;
+    const int r0 = lane_base + (lane >> 2);  // rows inside the tile
+    const int cq = 2 * (lane & 3);           // column offset inside a block
+    const uint32_t lane_off = (uint32_t)lane_base << 16;
+    const uint32_t d_addr = tmem_base + slot * G::SLOT_COLS + lane_off;
+    const uint32_t ahi_addr = d_addr + H;
+    const uint32_t alo_addr = d_addr + H + H / 2;
+    uint32_t d_use = 0;
+#ifdef GNN_TRACE
+    int tr_iter = 0;
+    const int trow = (hq == 0 && quarter == 2) ? r0 - 64 : -1;   // 0 for one thread of slot 0's first warp
+#endif
 
     auto arrive_a = [&]() {
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&a_full[slot]);
     };
-    auto wait_d = [&]() -> bool {
-      const bool ok = bounded_wait(&d_full[slot], d_use & 1, abort_flag, p.err);   // never early-exits a tile
+    auto wait_d = [&]() -> bool {            // never early-exits a tile
+      const bool ok = bounded_wait(&d_full[slot], d_use & 1, abort_flag, p.err);
       d_use++;
       tc_fence_after();
       return ok;
     };
-    auto load_d_add = [&](float* v) {        // v += D (this thread's HH columns)
-#pragma unroll
-      for (int c = 0; c < HH; c += 16) {
-        float t[16];
-        tmem_ld16(d_addr + c, t);
-        tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) v[c + i] += t[i];
-      }
+    auto quad_sum = [&](float x) {
+      x += __shfl_xor_sync(0xffffffffu, x, 1);
+      x += __shfl_xor_sync(0xffffffffu, x, 2);
+      return x;
     };
-    auto store_a = [&](const float* v) {     // split to bf16 hi/lo, write A operand
+    // Row-tiled state "T8": element (r, c) at ((r/128)*(H/8) + c/8)*1024 + (r%128)*8 + c%8.
+    auto t8 = [&](const float* base, int row, int b) -> const float2* {
+      return reinterpret_cast<const float2*>(base + (((size_t)(row >> 7) * NB + b) * 128 + (row & 127)) * 8 + cq);
+    };
+    auto rm = [&](const float* base, int row, int b) -> const float2* {   // row-major [*, H]
+      return reinterpret_cast<const float2*>(base + (size_t)row * H + 8 * b + cq);
+    };
+    auto load_d = [&](float* v) {            // D of both rows, one TMEM round trip
 #pragma unroll
-      for (int c = 0; c < HH; c += 16) {
-        uint32_t hi[8], lo[8];
+      for (int c = 0; c < H; c += 64) tmem_ld_16x256b_x8(d_addr + c, v + c / 2);
+      tmem_ld_wait();
+    };
+    auto put_a = [&](const float* v) {       // both rows -> bf16 hi/lo A operand
 #pragma unroll
-        for (int i = 0; i < 8; ++i) split_bf16x2(v[c + 2 * i], v[c + 2 * i + 1], hi[i], lo[i]);
-        tmem_st8(ahi_addr + c / 2, hi);
-        tmem_st8(alo_addr + c / 2, lo);
+      for (int h = 0; h < NB; h += 8) {
+        uint32_t hi[16], lo[16];
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+          split_bf16x2(v[4 * (h + b)], v[4 * (h + b) + 1], hi[2 * b], lo[2 * b]);
+          split_bf16x2(v[4 * (h + b) + 2], v[4 * (h + b) + 3], hi[2 * b + 1], lo[2 * b + 1]);
+        }
+        tmem_st_16x128b_x8(ahi_addr + 4 * h, hi);
+        tmem_st_16x128b_x8(alo_addr + 4 * h, lo);
       }
       tmem_st_wait();
     };
-    auto xchg = [&](float mine) -> float {   // value of the other column half of this row
-      float* b = red_slot + xbuf * 256;
-      b[half * 128 + trow] = mine;
-      named_bar_sync(1 + slot, 256);
-      const float other = b[(1 - half) * 128 + trow];
-      xbuf ^= 1;
-      return other;
-    };
-    auto ln_relu = [&](float* v, const float* gamma, const float* beta) {
-      float s = 0.f;
-#pragma unroll
-      for (int i = 0; i < HH; ++i) s += v[i];
-      s += xchg(s);
-      const float mean = s * (1.0f / H);
-      float q = 0.f;
-#pragma unroll
-      for (int i = 0; i < HH; ++i) { const float dd = v[i] - mean; q += dd * dd; }
-      q += xchg(q);
-      const float rstd = rsqrtf(q * (1.0f / H) + p.eps);
-#pragma unroll
-      for (int i = 0; i < HH; ++i) v[i] = fmaxf(fmaf((v[i] - mean) * rstd, gamma[c0 + i], beta[c0 + i]), 0.f);
-    };
     auto add_vec = [&](float* v, const float* b) {
 #pragma unroll
-      for (int i = 0; i < HH; ++i) v[i] += b[c0 + i];
-    };
-    auto load_row = [&](float* v, const float* base, bool ok) {   // v = base[c0 .. c0+HH)
-      if (ok) {
-        const float4* s4 = reinterpret_cast<const float4*>(base + c0);
-#pragma unroll
-        for (int i = 0; i < HH / 4; ++i) { const float4 t = s4[i]; v[4*i] = t.x; v[4*i+1] = t.y; v[4*i+2] = t.z; v[4*i+3] = t.w; }
-      } else {
-#pragma unroll
-        for (int i = 0; i < HH; ++i) v[i] = 0.f;
+      for (int k = 0; k < NB; ++k) {
+        const float2 t = *reinterpret_cast<const float2*>(b + 8 * k + cq);
+        v[4 * k] += t.x; v[4 * k + 1] += t.y; v[4 * k + 2] += t.x; v[4 * k + 3] += t.y;
       }
     };
-    auto add_row = [&](float* v, const float* base) {
-      const float4* s4 = reinterpret_cast<const float4*>(base + c0);
+    auto ln_relu = [&](float* v, const float* gamma, const float* beta) {
+      float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-      for (int i = 0; i < HH / 4; ++i) { const float4 t = s4[i]; v[4*i] += t.x; v[4*i+1] += t.y; v[4*i+2] += t.z; v[4*i+3] += t.w; }
-    };
-    auto store_row = [&](float* base, const float* v) {
-      float4* d4 = reinterpret_cast<float4*>(base + c0);
+      for (int k = 0; k < NB; ++k) { s0 += v[4 * k] + v[4 * k + 1]; s1 += v[4 * k + 2] + v[4 * k + 3]; }
+      const float m0 = quad_sum(s0) * (1.0f / H), m1 = quad_sum(s1) * (1.0f / H);
+      float q0 = 0.f, q1 = 0.f;
 #pragma unroll
-      for (int i = 0; i < HH / 4; ++i) d4[i] = make_float4(v[4*i], v[4*i+1], v[4*i+2], v[4*i+3]);
-    };
-    // First layer of an encoder on CUDA cores: v = W1 f + b1, W1 [H, nf] row-major in smem.
-    auto small_linear = [&](float* v, const float* f, int nf, const float* W1, const float* b1) {
-#pragma unroll
-      for (int i = 0; i < HH; ++i) {
-        float acc = b1[c0 + i];
-        for (int k = 0; k < nf; ++k) acc = fmaf(W1[(c0 + i) * nf + k], f[k], acc);
-        v[i] = acc;
+      for (int k = 0; k < NB; ++k) {
+        v[4 * k] -= m0; v[4 * k + 1] -= m0; v[4 * k + 2] -= m1; v[4 * k + 3] -= m1;
+        q0 = fmaf(v[4 * k], v[4 * k], fmaf(v[4 * k + 1], v[4 * k + 1], q0));
+        q1 = fmaf(v[4 * k + 2], v[4 * k + 2], fmaf(v[4 * k + 3], v[4 * k + 3], q1));
       }
+      const float i0 = rsqrtf(quad_sum(q0) * (1.0f / H) + p.eps);
+      const float i1 = rsqrtf(quad_sum(q1) * (1.0f / H) + p.eps);
+#pragma unroll
+      for (int k = 0; k < NB; ++k) {
+        const float2 g = *reinterpret_cast<const float2*>(gamma + 8 * k + cq);
+        const float2 b = *reinterpret_cast<const float2*>(beta + 8 * k + cq);
+        v[4 * k] = fmaxf(fmaf(v[4 * k] * i0, g.x, b.x), 0.f);
+        v[4 * k + 1] = fmaxf(fmaf(v[4 * k + 1] * i0, g.y, b.y), 0.f);
+        v[4 * k + 2] = fmaxf(fmaf(v[4 * k + 2] * i1, g.x, b.x), 0.f);
+        v[4 * k + 3] = fmaxf(fmaf(v[4 * k + 3] * i1, g.y, b.y), 0.f);
+      }
+    };
+    auto load_t8 = [&](float* v, const float* base, int row0, bool ok0, bool ok1) {
+#pragma unroll
+      for (int k = 0; k < NB; ++k) {
+        const float2 a = ok0 ? *t8(base, row0, k) : make_float2(0.f, 0.f);
+        const float2 b = ok1 ? *t8(base, row0 + 8, k) : make_float2(0.f, 0.f);
+        v[4 * k] = a.x; v[4 * k + 1] = a.y; v[4 * k + 2] = b.x; v[4 * k + 3] = b.y;
+      }
+    };
+    auto store_t8 = [&](float* base, int row0, bool ok0, bool ok1, const float* v) {
+#pragma unroll
+      for (int k = 0; k < NB; ++k) {
+        if (ok0) *const_cast<float2*>(t8(base, row0, k)) = make_float2(v[4 * k], v[4 * k + 1]);
+        if (ok1) *const_cast<float2*>(t8(base, row0 + 8, k)) = make_float2(v[4 * k + 2], v[4 * k + 3]);
+      }
+    };
+    // D (+ bias) of both rows streamed to a row-major output, 8 blocks per TMEM round trip.
+    auto stream_d = [&](float* base, int row0, bool ok0, bool ok1, const float* bias) {
+#pragma unroll
+      for (int c = 0; c < H; c += 64) {
+        float t[32];
+        tmem_ld_16x256b_x8(d_addr + c, t);
+        tmem_ld_wait();
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int kb = c / 8 + k;
+          float2 bb = make_float2(0.f, 0.f);
+          if (bias) bb = *reinterpret_cast<const float2*>(bias + 8 * kb + cq);
+          if (ok0) *const_cast<float2*>(rm(base, row0, kb)) = make_float2(t[4 * k] + bb.x, t[4 * k + 1] + bb.y);
+          if (ok1) *const_cast<float2*>(rm(base, row0 + 8, kb)) = make_float2(t[4 * k + 2] + bb.x, t[4 * k + 3] + bb.y);
+        }
+      }
+    };
+    auto prefetch_next_tile = [&](const float* base, int tile) {
+      const int nt = tile + 2 * (int)gridDim.x;
+      if (lane == 0 && wq == 0 && nt < p.n_tiles) prefetch_l2_bulk(base + (size_t)nt * kTileRows * H, kTileRows * H * 4);
     };
 
     const int L = p.n_layers;
@@ -298,131 +410,170 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     for (int pair = blockIdx.x; ok && pair < n_pairs; pair += gridDim.x) {
       const int tile = 2 * pair + slot;
       if (tile >= p.n_tiles) break;
-      const int row = tile * kTileRows + trow;
-      const bool valid = row < p.n_rows;
-      float v[HH];
+      const int row0 = tile * kTileRows + r0, row1 = row0 + 8;
+      const bool ok0 = row0 < p.n_rows, ok1 = row1 < p.n_rows;
+      float v[4 * NB];
 
       if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
         // vec layout: [gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]
-        load_row(v, p.e + (size_t)row * H, valid);
-        store_a(v); arrive_a();
-        // layer-1 pre-activation terms of the endpoints (P_d carries b1)
-        if (valid) {
-          const int s = p.src_sorted[row], d = p.dst_sorted[row];
-          load_row(v, p.ps + (size_t)s * H, true);
-          add_row(v, p.pd + (size_t)d * H);
-        } else {
+        if (slot == 0 && wq == 0 && lane == 0) progress[0] = pair;
+        GNN_TRACE_W(0);
+        load_t8(v, p.e, row0, ok0, ok1);
+        GNN_TRACE_W(1);
+        put_a(v);
+        arrive_a();                                     // job: D = e * W_e^T
+        GNN_TRACE_W(2);
+        // layer-1 terms of the endpoints, loaded while the MMA runs: P_s[src] + P_d[dst] (P_d carries b1)
+        {
+          const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
+          const int s1 = ok1 ? p.src_sorted[row1] : 0, d1 = ok1 ? p.dst_sorted[row1] : 0;
 #pragma unroll
-          for (int i = 0; i < HH; ++i) v[i] = 0.f;
-        }
-        for (int l = 1; l <= L; ++l) {
-          if (l > 1) {
-#pragma unroll
-            for (int i = 0; i < HH; ++i) v[i] = 0.f;
+          for (int k = 0; k < NB; ++k) {
+            const float2 a0 = *rm(p.ps, s0, k), b0 = *rm(p.pd, d0, k);
+            const float2 a1 = *rm(p.ps, s1, k), b1 = *rm(p.pd, d1, k);
+            v[4 * k] = a0.x + b0.x; v[4 * k + 1] = a0.y + b0.y;
+            v[4 * k + 2] = a1.x + b1.x; v[4 * k + 3] = a1.y + b1.y;
           }
+        }
+        GNN_TRACE_W(3);
+        ok &= wait_d();
+        GNN_TRACE_W(5);
+#pragma unroll
+        for (int c = 0; c < H; c += 64) {               // v += D
+          float t[32];
+          tmem_ld_16x256b_x8(d_addr + c, t);
+          tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[c / 2 + i] += t[i];
+        }
+        ln_relu(v, vecs, vecs + H);
+        if (L > 1) { put_a(v); arrive_a(); }
+        GNN_TRACE_W(6);
+        for (int l = 2; l <= L; ++l) {
           ok &= wait_d();
-          load_d_add(v);
-          const float* vb = vecs + (l == 1 ? 0 : (2 + 3 * (l - 2)) * H);
-          if (l > 1) { add_vec(v, vb); vb += H; }
-          ln_relu(v, vb, vb + H);
-          if (l < L) { store_a(v); arrive_a(); }
+          GNN_TRACE_W(5 + 2 * (l - 1));
+          load_d(v);
+          const float* vb = vecs + (2 + 3 * (l - 2)) * H;
+          add_vec(v, vb);
+          ln_relu(v, vb + H, vb + 2 * H);
+          if (l < L) { put_a(v); arrive_a(); }
+          GNN_TRACE_W(6 + 2 * (l - 1));
         }
         if constexpr (KIND == TileKind::EdgeUpdate) {
-          if (ok && valid) store_row(p.e + (size_t)row * H, v);
+          store_t8(p.e, row0, ok && ok0, ok && ok1, v);
+          GNN_TRACE_W(11);
         } else {
           const float* wo = vecs + (2 + 3 * (L - 1)) * H;
-          float z = 0.f;
+          float z0 = 0.f, z1 = 0.f;
 #pragma unroll
-          for (int i = 0; i < HH; ++i) z = fmaf(v[i], wo[c0 + i], z);
-          z += xchg(z);
-          if (ok && valid && half == 0) {
-            const float logit = z + wo[H];
-            const float sc = 1.0f / (1.0f + __expf(-logit));
-            const bool good = p.key_sorted[row] < p.n_nodes;
-            p.scores[p.perm[row]] = good ? sc : __int_as_float(0x7fc00000);
+          for (int k = 0; k < NB; ++k) {
+            const float2 w = *reinterpret_cast<const float2*>(wo + 8 * k + cq);
+            z0 = fmaf(v[4 * k], w.x, fmaf(v[4 * k + 1], w.y, z0));
+            z1 = fmaf(v[4 * k + 2], w.x, fmaf(v[4 * k + 3], w.y, z1));
+          }
+          z0 = quad_sum(z0) + wo[H];
+          z1 = quad_sum(z1) + wo[H];
+          if (ok && (lane & 3) == 0) {
+            const float nan = __int_as_float(0x7fc00000);
+            if (ok0) p.scores[p.perm[row0]] = p.key_sorted[row0] < p.n_nodes ? 1.0f / (1.0f + __expf(-z0)) : nan;
+            if (ok1) p.scores[p.perm[row1]] = p.key_sorted[row1] < p.n_nodes ? 1.0f / (1.0f + __expf(-z1)) : nan;
           }
         }
       } else if constexpr (KIND == TileKind::EdgeEncoder) {
-        // vec layout: [W1 (H x 2), b1, gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L]
-        float f[2] = {0.f, 0.f};
-        if (valid) {
-          const int s = p.src_sorted[row], d = p.dst_sorted[row];
-          const float* xs = p.x + (size_t)s * p.x_stride;
-          const float* xd = p.x + (size_t)d * p.x_stride;
-          f[0] = xd[0] - xs[0];
-          float dphi = xd[1] - xs[1];
-          if (dphi > 1.0f) dphi -= 2.0f;
-          if (dphi <= -1.0f) dphi += 2.0f;
-          f[1] = dphi;
-        }
-        const float* W1 = vecs;
-        const float* vb = vecs + 2 * H;
-        small_linear(v, f, 2, W1, vb);
-        ln_relu(v, vb + H, vb + 2 * H);
-        store_a(v); arrive_a();
-        for (int l = 2; l <= L; ++l) {
+        // vec layout: [W1^T (2 x H), b1, gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L]
+        float f[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
 #pragma unroll
-          for (int i = 0; i < HH; ++i) v[i] = 0.f;
+        for (int r = 0; r < 2; ++r) {
+          const int row = r ? row1 : row0;
+          if (r ? ok1 : ok0) {
+            const int s = p.src_sorted[row], d = p.dst_sorted[row];
+            const float* xs = p.x + (size_t)s * p.x_stride;
+            const float* xd = p.x + (size_t)d * p.x_stride;
+            f[r][0] = xd[0] - xs[0];
+            float dphi = xd[1] - xs[1];
+            if (dphi > 1.0f) dphi -= 2.0f;
+            if (dphi <= -1.0f) dphi += 2.0f;
+            f[r][1] = dphi;
+          }
+        }
+        const float* vb = vecs + 2 * H;
+#pragma unroll
+        for (int k = 0; k < NB; ++k) {
+          const float2 w0 = *reinterpret_cast<const float2*>(vecs + 8 * k + cq);
+          const float2 w1 = *reinterpret_cast<const float2*>(vecs + H + 8 * k + cq);
+          v[4 * k] = fmaf(w1.x, f[0][1], w0.x * f[0][0]);
+          v[4 * k + 1] = fmaf(w1.y, f[0][1], w0.y * f[0][0]);
+          v[4 * k + 2] = fmaf(w1.x, f[1][1], w0.x * f[1][0]);
+          v[4 * k + 3] = fmaf(w1.y, f[1][1], w0.y * f[1][0]);
+        }
+        add_vec(v, vb);
+        ln_relu(v, vb + H, vb + 2 * H);
+        put_a(v);
+        arrive_a();
+        for (int l = 2; l <= L; ++l) {
           ok &= wait_d();
-          load_d_add(v);
+          load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
           add_vec(v, vl);
           ln_relu(v, vl + H, vl + 2 * H);
-          if (l < L) { store_a(v); arrive_a(); }
+          if (l < L) { put_a(v); arrive_a(); }
         }
-        if (ok && valid) store_row(p.e + (size_t)row * H, v);
+        store_t8(p.e, row0, ok && ok0, ok && ok1, v);
       } else {
         // NodeEncoder / NodeUpdate.
-        // vec layout: [W1 (H x n_feat) if encoder], (b_l, gamma_l, beta_l) for l = 1..L, b1_edge
+        // vec layout: [W1^T (n_feat x H) if encoder], (b_l, gamma_l, beta_l) for l = 1..L, b1_edge
         const float* vb = vecs + (KIND == TileKind::NodeEncoder ? p.n_feat * H : 0);
         int l0;
         if constexpr (KIND == TileKind::NodeEncoder) {
-          float f[16];
-          for (int k = 0; k < 16; ++k) f[k] = (valid && k < p.n_feat) ? p.x[(size_t)row * p.x_stride + k] : 0.f;
-          small_linear(v, f, p.n_feat, vecs, vb);
+#pragma unroll
+          for (int i = 0; i < 4 * NB; ++i) v[i] = 0.f;
+          for (int k = 0; k < p.n_feat; ++k) {          // layer 1 on CUDA cores
+            const float x0 = ok0 ? p.x[(size_t)row0 * p.x_stride + k] : 0.f;
+            const float x1 = ok1 ? p.x[(size_t)row1 * p.x_stride + k] : 0.f;
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+              const float2 w = *reinterpret_cast<const float2*>(vecs + k * H + 8 * b + cq);
+              v[4 * b] = fmaf(w.x, x0, v[4 * b]); v[4 * b + 1] = fmaf(w.y, x0, v[4 * b + 1]);
+              v[4 * b + 2] = fmaf(w.x, x1, v[4 * b + 2]); v[4 * b + 3] = fmaf(w.y, x1, v[4 * b + 3]);
+            }
+          }
+          add_vec(v, vb);
           ln_relu(v, vb + H, vb + 2 * H);
-          store_a(v); arrive_a();
+          put_a(v);
+          arrive_a();
           l0 = 2;
         } else {
-          load_row(v, p.h + (size_t)row * H, valid);
-          store_a(v); arrive_a();                       // job: D = h * W_nh^T
-#pragma unroll
-          for (int i = 0; i < HH; ++i) v[i] = 0.f;
-          if (valid) {                                  // a_j: CSR segment sum, fixed order
-            const int k0 = p.rowptr[row], k1 = p.rowptr[row + 1];
-            for (int k = k0; k < k1; ++k) add_row(v, p.e + (size_t)k * H);
-          }
-          ok &= wait_d();                // A free again
-          store_a(v); arrive_a();                       // job: D += a * W_na^T
+          load_t8(v, p.h, row0, ok0, ok1);
+          put_a(v);
+          arrive_a();                                   // job: D = h * W_h^T
+          prefetch_next_tile(p.h, tile);
+          prefetch_next_tile(p.agg, tile);
+          load_t8(v, p.agg, row0, ok0, ok1);            // a_j, summed by the aggregation kernel
+          ok &= wait_d();                               // A free again
+          put_a(v);
+          arrive_a();                                   // job: D += a * W_a^T
           l0 = 1;
         }
         for (int l = l0; l <= L; ++l) {
-#pragma unroll
-          for (int i = 0; i < HH; ++i) v[i] = 0.f;
           ok &= wait_d();
-          load_d_add(v);
+          load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
           add_vec(v, vl);
           ln_relu(v, vl + H, vl + 2 * H);
-          store_a(v); arrive_a();                       // next layer, or the P_s job
+          put_a(v);
+          arrive_a();                                   // next layer, or the P_s job
         }
-        if (ok && valid) store_row(p.h + (size_t)row * H, v);
-        // P_s = W_s h (no bias)
-#pragma unroll
-        for (int i = 0; i < HH; ++i) v[i] = 0.f;
-        ok &= wait_d();
-        load_d_add(v);
-        if (ok && valid) store_row(p.ps + (size_t)row * H, v);
+        store_t8(p.h, row0, ok && ok0, ok && ok1, v);   // new node state
+        ok &= wait_d();                                 // P_s = W_s h (no bias)
+        stream_d(p.ps, row0, ok && ok0, ok && ok1, nullptr);
         arrive_a();                                     // D read; A (= h) unchanged -> P_d job
-        // P_d = W_d h + b1 (edge-side bias)
-#pragma unroll
-        for (int i = 0; i < HH; ++i) v[i] = 0.f;
-        ok &= wait_d();
-        load_d_add(v);
-        add_vec(v, vb + 3 * L * H);
-        if (ok && valid) store_row(p.pd + (size_t)row * H, v);
+        ok &= wait_d();                                 // P_d = W_d h + b1 (edge-side bias)
+        stream_d(p.pd, row0, ok && ok0, ok && ok1, vb + 3 * L * H);
       }
       if (!ok) break;                        // leave only between tiles
+#ifdef GNN_TRACE
+      ++tr_iter;
+#endif
     }
     __syncwarp();
   }
@@ -434,6 +585,41 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     tc_fence_after();
     tmem_dealloc(tmem_base, G::TMEM_COLS);
   }
+}
+
+// a_j = sum of the messages m_ij of the edges into node j (CSR segment of j,
+// fixed slot order, no atomics).  One thread per (node, 8-column block): a
+// warp covers 32 consecutive nodes and one block, so both its loads (rows of
+// neighbouring segments, 32 bytes each) and its stores are contiguous.
+template <int H>
+__global__ void __launch_bounds__(256) aggregate_kernel(const float* __restrict__ e, const int* __restrict__ rowptr,
+                                                        int n_nodes, float* __restrict__ agg) {
+  constexpr int NB = H / 8;
+  const int b = blockIdx.y * 8 + (threadIdx.x >> 5);
+  const int j = blockIdx.x * 32 + (threadIdx.x & 31);
+  if (j >= n_nodes || b >= NB) return;
+  const int k0 = rowptr[j], k1 = rowptr[j + 1];
+  auto row = [&](int k) { return reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NB + b) * 128 + (k & 127)) * 8); };
+  float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0;
+  int k = k0;
+  for (; k + 4 <= k1; k += 4) {              // four rows in flight, summed in slot order
+    float4 x[4], y[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) { x[u] = row(k + u)[0]; y[u] = row(k + u)[1]; }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      a0.x += x[u].x; a0.y += x[u].y; a0.z += x[u].z; a0.w += x[u].w;
+      a1.x += y[u].x; a1.y += y[u].y; a1.z += y[u].z; a1.w += y[u].w;
+    }
+  }
+  for (; k < k1; ++k) {
+    const float4 x = row(k)[0], y = row(k)[1];
+    a0.x += x.x; a0.y += x.y; a0.z += x.z; a0.w += x.w;
+    a1.x += y.x; a1.y += y.y; a1.z += y.z; a1.w += y.w;
+  }
+  float4* o = reinterpret_cast<float4*>(agg + (((size_t)(j >> 7) * NB + b) * 128 + (j & 127)) * 8);
+  o[0] = a0;
+  o[1] = a1;
 }
 
 }  // namespace gnn

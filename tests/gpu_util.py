@@ -40,3 +40,10 @@ def check_parity(s_gpu, W, x, ei, T, tol=LOGIT_TOL_FP32, eps=1e-5):
     sure = np.abs(want) > DECISION_MARGIN
     assert np.array_equal(got[sure] > 0, want[sure] > 0), "edge decision mismatch"
     return float(err.max())
+
+
+def untile(buf, n_rows, H):
+    """Row-tiled state [R/128][H/8][128][8] -> row-major [n_rows, H]."""
+    R = (n_rows + 127) // 128 * 128
+    a = np.asarray(buf).reshape(R // 128, H // 8, 128, 8).transpose(0, 2, 1, 3).reshape(R, H)
+    return a[:n_rows]

@@ -8,7 +8,7 @@ import pytest
 
 from oracle import gnn_oracle as O
 from paper_2402_09633_gb300 import synthetic as S
-from tests.gpu_util import check_parity, run_gpu
+from tests.gpu_util import check_parity, run_gpu, untile
 
 pytestmark = pytest.mark.gpu
 
@@ -49,7 +49,8 @@ def test_node_state_after_iterations():
     W = S.init_weights(cfg, 3)
     x, ei = S.generate_event(S.EventSpec(3000, 9, "powerlaw", 0.02, n_edges=10007), 2)
     s, rc, net = run_gpu(cfg, W, x, ei, return_net=True)
-    h = net.debug_copy(3, (x.shape[0], 128), torch.float32).cpu().numpy()
+    R = (x.shape[0] + 127) // 128 * 128
+    h = untile(net.debug_copy(3, (R * 128,), torch.float32).cpu().numpy(), x.shape[0], 128)
     net.close()
     _, _, st = O.forward(W, x, ei, cfg.n_iters, return_logits=True, return_states=True)
     assert np.abs(h - st["h"]).max() < 2e-3
