@@ -171,6 +171,41 @@ const char* gnn_error_string(int code);
  */
 int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_t stream);
 
+/*
+ * gnn_csr_build_noalloc -- the destination-keyed CSR of an edge list, built
+ * without allocating any device memory.  (Library plumbing: the paper has no
+ * counterpart.)  It is for callers that must not allocate: a serving backend
+ * or host framework whose memory planner owns every device allocation and
+ * forbids new ones after start-up, or code that must keep cudaMalloc and
+ * cudaFree (and their implicit device synchronisation) off its request path.
+ *
+ * Scratch is one fixed, library-owned device array of
+ * GNN_CSR_NOALLOC_SCRATCH_BYTES bytes, allocated when the library is loaded
+ * on a device and held by every device that loads the library until the
+ * process exits.  The caller provides only inputs and outputs:
+ *   edge_index device int32 [2, n_edges] (row 0 sources, row 1 destinations)
+ *   rowptr     device int32 [n_nodes + 1]: first sorted slot of each node
+ *   perm       device int32 [n_edges]: input edge id of each sorted slot
+ *   src_sorted device int32 [n_edges]: source of each sorted slot
+ * The result is bit-identical to the CSR gnn_infer builds: edges stably
+ * sorted by destination (ties keep input order).  Edges with an endpoint
+ * outside [0, n_nodes) are placed after rowptr[n_nodes] (so rowptr[n_nodes]
+ * < n_edges reveals them) with source 0.
+ * Limits: n_edges <= GNN_CSR_NOALLOC_MAX_EDGES and 0 <= n_nodes < INT32_MAX;
+ * larger sizes, negative sizes or null pointers return GNN_ERR_INVALID_ARG
+ * before any device work.  The first call on a device looks up the scratch
+ * array's device address (device set-up; make that first call outside any
+ * stream capture).  All calls share the one array and it keeps the last
+ * call's contents (nothing in it needs to start at zero); calls that overlap
+ * on the GPU (several streams, or several host threads) race on it and must
+ * be serialised by the caller.  Enqueued on `stream`; no host synchronisation.
+ * Errors: INVALID_ARG, CUDA.
+ */
+#define GNN_CSR_NOALLOC_MAX_EDGES (1 << 20)
+#define GNN_CSR_NOALLOC_SCRATCH_BYTES (5u * 4u * GNN_CSR_NOALLOC_MAX_EDGES + 4u * 256u * 256u)
+int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes, int64_t n_edges, int32_t* rowptr,
+                          int32_t* perm, int32_t* src_sorted, gnn_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -17,6 +17,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -583,3 +584,89 @@ int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free CSR build: the radix-sort scratch lives in one file-scope
+// device array instead of context workspace.  Layout (int32 words):
+// keys_a | keys_b | vals_a | vals_b | src_clamped (GNN_CSR_NOALLOC_MAX_EDGES
+// each) | per-tile digit histograms (256 x 256).  Host code must not use the
+// array's name as a device address: the address comes from
+// cudaGetSymbolAddress, looked up once per device with that device current.
+static_assert((GNN_CSR_NOALLOC_MAX_EDGES + kRadixTile - 1) / kRadixTile <= 256, "histogram area too small");
+static __device__ __align__(256) unsigned char g_csr_noalloc_scratch[GNN_CSR_NOALLOC_SCRATCH_BYTES];
+static __device__ uint32_t g_csr_noalloc_err;
+
+namespace {
+constexpr int kNoallocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+unsigned char* g_noalloc_scratch_dev[kNoallocMaxDevices] = {};
+uint32_t* g_noalloc_err_dev[kNoallocMaxDevices] = {};
+
+// Device addresses of the scratch array and error word on the current device.
+cudaError_t noalloc_setup(unsigned char** scratch, uint32_t** err) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kNoallocMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_scratch_dev[dev]) {
+    void* sp = nullptr;
+    void* ep = nullptr;
+    e = cudaGetSymbolAddress(&sp, g_csr_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    e = cudaGetSymbolAddress(&ep, g_csr_noalloc_err);
+    if (e != cudaSuccess) return e;
+    g_noalloc_scratch_dev[dev] = static_cast<unsigned char*>(sp);
+    g_noalloc_err_dev[dev] = static_cast<uint32_t*>(ep);
+  }
+  *scratch = g_noalloc_scratch_dev[dev];
+  *err = g_noalloc_err_dev[dev];
+  return cudaSuccess;
+}
+}  // namespace
+
+extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes, int64_t n_edges,
+                                     int32_t* rowptr, int32_t* perm, int32_t* src_sorted, gnn_stream_t stream) {
+  if (n_nodes < 0 || n_nodes >= INT32_MAX || n_edges < 0 || n_edges > GNN_CSR_NOALLOC_MAX_EDGES || !rowptr)
+    return GNN_ERR_INVALID_ARG;
+  if (n_edges > 0 && (!edge_index || !perm || !src_sorted)) return GNN_ERR_INVALID_ARG;
+  unsigned char* scratch = nullptr;
+  uint32_t* err = nullptr;
+  cudaError_t ce = noalloc_setup(&scratch, &err);
+  if (ce != cudaSuccess) return cuda_fail(ce);
+  cudaStream_t st = (cudaStream_t)stream;
+  const int N = (int)n_nodes, E = (int)n_edges;
+  const int tb = 256;
+  if (E == 0) {                                   // every row pointer is 0
+    csr_rowptr_kernel<<<1, tb, 0, st>>>(nullptr, 0, N, rowptr);
+    ce = cudaGetLastError();
+    return ce == cudaSuccess ? GNN_OK : cuda_fail(ce);
+  }
+  int* words = reinterpret_cast<int*>(scratch);
+  int* keys_a = words;
+  int* keys_b = keys_a + GNN_CSR_NOALLOC_MAX_EDGES;
+  int* vals_a = keys_b + GNN_CSR_NOALLOC_MAX_EDGES;
+  int* vals_b = vals_a + GNN_CSR_NOALLOC_MAX_EDGES;
+  int* src_c = vals_b + GNN_CSR_NOALLOC_MAX_EDGES;
+  int* hist = src_c + GNN_CSR_NOALLOC_MAX_EDGES;
+  csr_keys_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(edge_index, E, N, keys_a, vals_a, src_c, err);
+  int bits = 0;
+  while (bits < 31 && (N >> bits) != 0) ++bits;   // keys lie in [0, N]
+  if (bits == 0) bits = 1;
+  const int passes = (bits + 7) / 8;
+  const int tiles = (E + kRadixTile - 1) / kRadixTile;
+  int *kin = keys_a, *vin = vals_a, *kout = keys_b, *vout = vals_b;
+  for (int ps = 0; ps < passes; ++ps) {
+    const int shift = 8 * ps;
+    radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, E, shift, tiles, hist);
+    exclusive_scan_kernel<<<1, 1024, 0, st>>>(hist, 256 * tiles);
+    radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, E, shift, tiles, hist);
+    int* t = kin; kin = kout; kout = t;
+    t = vin; vin = vout; vout = t;
+  }
+  // sorted keys in kin; kout is free and receives the (unused) clamped destinations
+  csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, src_c, E, N, perm, src_sorted, kout);
+  csr_rowptr_kernel<<<(E + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, rowptr);
+  ce = cudaGetLastError();
+  return ce == cudaSuccess ? GNN_OK : cuda_fail(ce);
+}
