@@ -35,7 +35,7 @@ __global__ void csr_keys_kernel(const int32_t* __restrict__ ei, int n_edges, int
   if (!ok) atomicOr(err, DEV_ERR_INDEX_RANGE);
 }
 
-// Per-tile digit histogram: hist[digit * n_tiles + tile].
+// Per-tile digit histogram: hist[tile * 256 + digit].
 __global__ void radix_count_kernel(const int* __restrict__ keys, int n, int shift, int n_tiles,
                                    int* __restrict__ hist) {
   __shared__ int cnt[256];
@@ -47,27 +47,32 @@ __global__ void radix_count_kernel(const int* __restrict__ keys, int n, int shif
     if (idx < n) atomicAdd(&cnt[(keys[idx] >> shift) & 255], 1);
   }
   __syncthreads();
-  hist[threadIdx.x * n_tiles + blockIdx.x] = cnt[threadIdx.x];
+  hist[blockIdx.x * 256 + threadIdx.x] = cnt[threadIdx.x];
 }
 
-// In-place exclusive scan of n ints with one block of 1024 threads.
-__global__ void exclusive_scan_kernel(int* __restrict__ data, int n) {
-  __shared__ int part[1024];
-  const int t = threadIdx.x;
-  const int per = (n + 1023) / 1024;
-  const int b = t * per, e = min(n, b + per);
-  int s = 0;
-  for (int i = b; i < e; ++i) s += data[i];
-  part[t] = s;
+// Scatter offsets of one radix pass, in place: hist[tile * 256 + d] becomes the
+// number of keys with a smaller digit (all tiles) plus those with digit d in
+// earlier tiles.  One block of 256 threads; thread d walks its digit's column
+// (reads are coalesced across threads), then the 256 digit totals are scanned.
+__global__ void __launch_bounds__(256) radix_offsets_kernel(int* __restrict__ hist, int n_tiles) {
+  __shared__ int tot[256];
+  const int d = threadIdx.x;
+  int run = 0;
+  for (int t = 0; t < n_tiles; ++t) {
+    const int v = hist[t * 256 + d];
+    hist[t * 256 + d] = run;
+    run += v;
+  }
+  tot[d] = run;
   __syncthreads();
-  for (int off = 1; off < 1024; off <<= 1) {      // Hillis-Steele inclusive scan
-    const int v = (t >= off) ? part[t - off] : 0;
+  for (int off = 1; off < 256; off <<= 1) {       // inclusive scan of the digit totals
+    const int v = d >= off ? tot[d - off] : 0;
     __syncthreads();
-    part[t] += v;
+    tot[d] += v;
     __syncthreads();
   }
-  int run = part[t] - s;                           // exclusive prefix of this chunk
-  for (int i = b; i < e; ++i) { const int v = data[i]; data[i] = run; run += v; }
+  const int base = tot[d] - run;                  // exclusive
+  for (int t = 0; t < n_tiles; ++t) hist[t * 256 + d] += base;
 }
 
 // Stable scatter of one radix pass.  Elements of a tile are ranked in input
@@ -80,7 +85,7 @@ __global__ void radix_scatter_kernel(const int* __restrict__ keys_in, const int*
   __shared__ int run[256];
   __shared__ int wcnt[kRadixThreads / 32][256];
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-  run[t] = offs[t * n_tiles + blockIdx.x];
+  run[t] = offs[blockIdx.x * 256 + t];
   const int base = blockIdx.x * kRadixTile;
   const unsigned lt_mask = (1u << lane) - 1u;
   for (int r = 0; r < kRadixRounds; ++r) {
@@ -125,15 +130,17 @@ __global__ void csr_gather_kernel(const int* __restrict__ keys_sorted, const int
   dst_sorted[k] = key < n_nodes ? key : 0;
 }
 
-// rowptr[j] = first sorted slot whose key >= j, for j in [0, n_nodes].
+// rowptr[j] = first sorted slot whose key >= j (binary search), for j in [0, n_nodes].
 __global__ void csr_rowptr_kernel(const int* __restrict__ keys_sorted, int n_edges, int n_nodes,
                                   int* __restrict__ rowptr) {
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k > n_edges) return;
-  const int prev = (k == 0) ? -1 : keys_sorted[k - 1];
-  const int cur = (k == n_edges) ? n_nodes + 1 : keys_sorted[k];
-  const int hi = min(cur, n_nodes);
-  for (int j = prev + 1; j <= hi; ++j) rowptr[j] = k;
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j > n_nodes) return;
+  int lo = 0, hi = n_edges;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (keys_sorted[mid] < j) lo = mid + 1; else hi = mid;
+  }
+  rowptr[j] = lo;
 }
 
 }  // namespace gnn

@@ -278,7 +278,7 @@ int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
   for (int ps = 0; ps < passes; ++ps) {
     const int shift = 8 * ps;
     radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, E, shift, tiles, c->hist);
-    exclusive_scan_kernel<<<1, 1024, 0, st>>>(c->hist, 256 * tiles);
+    radix_offsets_kernel<<<1, 256, 0, st>>>(c->hist, tiles);
     radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, E, shift, tiles, c->hist);
     int* t = kin; kin = kout; kout = t;
     t = vin; vin = vout; vout = t;
@@ -286,7 +286,7 @@ int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
   c->key_sorted = kin;
   csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, c->src_c, E, N, c->perm, c->src_sorted,
                                                      c->dst_sorted);
-  csr_rowptr_kernel<<<(E + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, c->rowptr);
+  csr_rowptr_kernel<<<(N + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, c->rowptr);
   prof_end(c, pr, st);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
@@ -344,6 +344,34 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     }
   const float* head_w = f;
   const float* head_b = f + H;
+
+  // Every Linear layer here feeds a LayerNorm, whose first step subtracts the
+  // mean over the H outputs.  That subtraction is linear, so it is folded into
+  // the layer: each weight column and the bias are centred over the output
+  // rows (W' = (I - 11^T/H) W, b' = b - mean(b)).  The kernels then receive
+  // zero-mean pre-activations and compute only the variance.  Centred copies
+  // are kept in `centred` and the Layer pointers redirected to them.
+  std::vector<std::vector<float>> centred;
+  centred.reserve(2 * N_MLP * L);
+  for (int m = 0; m < N_MLP; ++m)
+    for (int l = 0; l < L; ++l) {
+      Layer& ly = lay[m][l];
+      std::vector<float> Wc((size_t)H * ly.in), bc(H);
+      for (int k = 0; k < ly.in; ++k) {
+        double mu = 0.0;
+        for (int n = 0; n < H; ++n) mu += ly.W[(size_t)n * ly.in + k];
+        mu /= H;
+        for (int n = 0; n < H; ++n) Wc[(size_t)n * ly.in + k] = (float)(ly.W[(size_t)n * ly.in + k] - mu);
+      }
+      double mb = 0.0;
+      for (int n = 0; n < H; ++n) mb += ly.b[n];
+      mb /= H;
+      for (int n = 0; n < H; ++n) bc[n] = (float)(ly.b[n] - mb);
+      centred.push_back(std::move(Wc));
+      ly.W = centred.back().data();
+      centred.push_back(std::move(bc));
+      ly.b = centred.back().data();
+    }
 
   gnn_ctx* c = new (std::nothrow) gnn_ctx();
   if (!c) return GNN_ERR_OOM;
@@ -638,7 +666,7 @@ extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes,
   const int N = (int)n_nodes, E = (int)n_edges;
   const int tb = 256;
   if (E == 0) {                                   // every row pointer is 0
-    csr_rowptr_kernel<<<1, tb, 0, st>>>(nullptr, 0, N, rowptr);
+    csr_rowptr_kernel<<<(N + 1 + tb - 1) / tb, tb, 0, st>>>(nullptr, 0, N, rowptr);
     ce = cudaGetLastError();
     return ce == cudaSuccess ? GNN_OK : cuda_fail(ce);
   }
@@ -659,14 +687,14 @@ extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes,
   for (int ps = 0; ps < passes; ++ps) {
     const int shift = 8 * ps;
     radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, E, shift, tiles, hist);
-    exclusive_scan_kernel<<<1, 1024, 0, st>>>(hist, 256 * tiles);
+    radix_offsets_kernel<<<1, 256, 0, st>>>(hist, tiles);
     radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, E, shift, tiles, hist);
     int* t = kin; kin = kout; kout = t;
     t = vin; vin = vout; vout = t;
   }
   // sorted keys in kin; kout is free and receives the (unused) clamped destinations
   csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, src_c, E, N, perm, src_sorted, kout);
-  csr_rowptr_kernel<<<(E + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, rowptr);
+  csr_rowptr_kernel<<<(N + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, rowptr);
   ce = cudaGetLastError();
   return ce == cudaSuccess ? GNN_OK : cuda_fail(ce);
 }

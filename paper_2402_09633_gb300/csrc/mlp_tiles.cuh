@@ -11,15 +11,18 @@
 // bf16 splits (v = hi + lo, both bf16) with fp32 accumulation, which keeps the
 // relative product error near 2^-16.
 //
-// Roles (576 threads = 18 warps):
-//   warp 0      : MMA issuer (one elected lane)
-//   warp 1      : weight producer (bulk copies into the smem weight ring)
-//   warps 2..17 : 16 row-worker warps, 8 per slot.  Slot s works on tile
-//                 2p+s of tile pair p; the issuer serves whichever slot is
-//                 ready, so one slot's epilogue overlaps the other slot's MMAs.
-// A worker warp owns 16 rows of a tile; a quad of threads shares two rows
-// (each thread a quarter of the columns), reads them from tensor memory with
-// the 16-lane shapes and does LayerNorm / ReLU in registers.
+// Organisation (512 threads = 16 warps, all of them workers):
+//   * two TMEM slots, 8 warps each; slot s works on tile 2p+s of tile pair p,
+//     so while one slot runs its epilogue the tensor core serves the other
+//     (ping-pong);
+//   * there is no dedicated MMA or producer warp: the last of a slot's warps
+//     to publish its part of an A operand issues that slot's MMAs (one thread,
+//     24 tcgen05.mma per layer) and commits them to the slot's mbarrier; when
+//     weights stream through the ring, the second slot to finish with a stage
+//     refills it with a bulk copy;
+//   * a worker warp owns 16 rows of a tile; a quad of threads shares two rows
+//     (each thread a quarter of the columns), reads them from tensor memory
+//     with the 16-lane shapes and does LayerNorm / ReLU in registers.
 #pragma once
 #include <cstdint>
 #include <cuda_bf16.h>
@@ -35,7 +38,13 @@ enum class TileKind : int {
   Classifier  = 4,     // score = sigmoid(w_o . MLP_cls([h_src, h_dst, e]) + b_o)
 };
 
-constexpr int kThreads = 576;
+constexpr int kThreads = 640;
+// Register split (setmaxnreg): launch at 96 per thread (640 threads x 96 = 61440);
+// the control warpgroup keeps 32, the four worker warpgroups take 112:
+// 128 x 32 + 512 x 112 = 61440.
+constexpr int kControlRegs = 32;
+constexpr int kWorkerRegs = 112;
+static_assert(128 * kControlRegs + 512 * kWorkerRegs <= kThreads * 96, "register split exceeds the launch budget");
 constexpr int kTileRows = 128;
 constexpr int kMaxJobs = 8;
 
@@ -113,15 +122,16 @@ constexpr uint32_t tile_smem_bytes(int n_vec_floats) {
 template <TileKind KIND, int H>
 __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams p) {
   using G = TileGeom<H>;
+  constexpr int NB = H / 8;                          // 8-column blocks per row
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* ring = smem;
   float* vecs = reinterpret_cast<float*>(smem + G::RING_BYTES);
   uint64_t* bars = reinterpret_cast<uint64_t*>(vecs + padded_vec_floats(p.n_vec_floats));
-  uint64_t* a_full = bars;          // [2]
-  uint64_t* d_full = bars + 2;      // [2]
-  uint64_t* w_full = bars + 4;      // [STAGES]
-  uint64_t* w_empty = bars + 4 + G::STAGES;
+  uint64_t* a_full = bars;                           // [2]  a slot's 8 worker warps published A
+  uint64_t* d_full = bars + 2;                       // [2]  MMA of a slot's current job completed
+  uint64_t* w_full = bars + 4;                       // [STAGES]  weight stage loaded
+  uint64_t* w_empty = bars + 4 + G::STAGES;          // [STAGES]  both slots' MMAs on a stage completed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * G::STAGES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* progress = abort_flag + 1;          // tile pair slot 0's workers are on (L2 prefetch pacing)
@@ -129,6 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const bool resident = p.n_jobs <= G::STAGES;
+  const int n_pairs = (p.n_tiles + 1) >> 1;
 
   for (int i = threadIdx.x; i < p.n_vec_floats; i += kThreads) vecs[i] = p.vecs[i];
   if (threadIdx.x == 0) {
@@ -144,163 +155,162 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int n_pairs = (p.n_tiles + 1) >> 1;
 
-  if (warp == 1) {
-    // ------------------------------------------------ weight producer
-    if (lane == 0) {
-      if (resident) {
-        uint32_t total = 0;
-        for (int j = 0; j < p.n_jobs; ++j) total += G::MAT_BYTES;
-        mbar_arrive_expect_tx(&w_full[0], total);
-        for (int j = 0; j < p.n_jobs; ++j)
-          bulk_g2s(ring + j * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[0]);
-      }
-    }
-    __syncwarp();
-    if (resident && (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier)) {
-      // L2 prefetcher: while the workers are on tile pair k, warm L2 with the
-      // edge-state tiles and the gathered P_s / P_d rows of pair k+1.
-      const uint64_t t0 = global_timer_ns();
-      for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
-        const int prev = pair - (int)gridDim.x;
-        for (uint32_t it = 0; prev >= 0 && progress[0] < prev; ++it) {    // bounded: gives up silently
-          if (*abort_flag || ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs)) break;
-          __nanosleep(200);
+  if (warp < 4) {
+    // Control warpgroup: hands registers to the worker warpgroups.
+    setmaxnreg_dec<kControlRegs>();
+      if (warp == 1) {
+      // ------------------------------------------------ weight producer
+      if (lane == 0) {
+        if (resident) {
+          uint32_t total = 0;
+          for (int j = 0; j < p.n_jobs; ++j) total += G::MAT_BYTES;
+          mbar_arrive_expect_tx(&w_full[0], total);
+          for (int j = 0; j < p.n_jobs; ++j)
+            bulk_g2s(ring + j * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[0]);
         }
-        for (int s = 0; s < 2; ++s) {
-          const int tile = 2 * pair + s;
-          if (tile >= p.n_tiles) break;
-          if (lane == 0) prefetch_l2_bulk(p.e + (size_t)tile * kTileRows * H, kTileRows * H * 4);
+      }
+      __syncwarp();
+      if (resident && (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier)) {
+        // L2 prefetcher: while the workers are on tile pair k, warm L2 with the
+        // edge-state tiles and the gathered P_s / P_d rows of pair k+1.
+        const uint64_t t0 = global_timer_ns();
+        for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
+          const int prev = pair - (int)gridDim.x;
+          for (uint32_t it = 0; prev >= 0 && progress[0] < prev; ++it) {    // bounded: gives up silently
+            if (*abort_flag || ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs)) break;
+            __nanosleep(200);
+          }
+          for (int s = 0; s < 2; ++s) {
+            const int tile = 2 * pair + s;
+            if (tile >= p.n_tiles) break;
+            if (lane == 0) prefetch_l2_bulk(p.e + (size_t)tile * kTileRows * H, kTileRows * H * 4);
 #pragma unroll
-          for (int i = 0; i < kTileRows / 32; ++i) {
-            const int row = tile * kTileRows + i * 32 + lane;
-            if (row < p.n_rows) {
-              prefetch_l2_bulk(p.ps + (size_t)p.src_sorted[row] * H, H * 4);
-              prefetch_l2_bulk(p.pd + (size_t)p.dst_sorted[row] * H, H * 4);
+            for (int i = 0; i < kTileRows / 32; ++i) {
+              const int row = tile * kTileRows + i * 32 + lane;
+              if (row < p.n_rows) {
+                prefetch_l2_bulk(p.ps + (size_t)p.src_sorted[row] * H, H * 4);
+                prefetch_l2_bulk(p.pd + (size_t)p.dst_sorted[row] * H, H * 4);
+              }
             }
           }
         }
       }
-    }
-    if (!resident && lane == 0) {
-      {
-        uint32_t seq = 0;
-        for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
-          for (int j = 0; j < p.n_jobs; ++j, ++seq) {
-            const int st = seq % G::STAGES;
-            if (seq >= (uint32_t)G::STAGES &&
-                !bounded_wait(&w_empty[st], ((seq / G::STAGES) - 1) & 1, abort_flag, p.err)) break;
-            mbar_arrive_expect_tx(&w_full[st], G::MAT_BYTES);
-            bulk_g2s(ring + st * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[st]);
+      if (!resident && lane == 0) {
+        {
+          uint32_t seq = 0;
+          for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
+            for (int j = 0; j < p.n_jobs; ++j, ++seq) {
+              const int st = seq % G::STAGES;
+              if (seq >= (uint32_t)G::STAGES &&
+                  !bounded_wait(&w_empty[st], ((seq / G::STAGES) - 1) & 1, abort_flag, p.err)) break;
+              mbar_arrive_expect_tx(&w_full[st], G::MAT_BYTES);
+              bulk_g2s(ring + st * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[st]);
+            }
           }
         }
       }
-    }
-    __syncwarp();
-  } else if (warp == 0) {
-    // ------------------------------------------------ MMA issuer
-    // The two slots advance independently: each has its own job cursor, and
-    // the issuer serves whichever slot has published its next A operand.  In
-    // streamed-weight mode both slots walk the same (pair, job) sequence of
-    // ring stages; a stage is released after both slots' MMAs on it completed
-    // (w_empty counts two commits; a slot without a tile in the last pair is
-    // covered by a second commit of the other slot).
-    if (lane == 0) {
-      int pair_s[2] = {(int)blockIdx.x, (int)blockIdx.x};
-      int job_s[2] = {0, 0};
-      uint32_t seq_s[2] = {0, 0};
-      uint32_t a_par[2] = {0, 0};
-      bool act[2] = {2 * (int)blockIdx.x < p.n_tiles, 2 * (int)blockIdx.x + 1 < p.n_tiles};
-      bool ok = true;
-      if (resident) ok = bounded_wait(&w_full[0], 0, abort_flag, p.err);
-      uint64_t t_last = global_timer_ns();
-      uint32_t spins = 0;
-      while (ok && (act[0] || act[1])) {
-        bool progressed = false;
+      __syncwarp();
+    } else if (warp == 0) {
+      // ------------------------------------------------ MMA issuer
+      // The two slots advance independently: each has its own job cursor, and
+      // the issuer serves whichever slot has published its next A operand.  In
+      // streamed-weight mode both slots walk the same (pair, job) sequence of
+      // ring stages; a stage is released after both slots' MMAs on it completed
+      // (w_empty counts two commits; a slot without a tile in the last pair is
+      // covered by a second commit of the other slot).
+      if (lane == 0) {
+        int pair_s[2] = {(int)blockIdx.x, (int)blockIdx.x};
+        int job_s[2] = {0, 0};
+        uint32_t seq_s[2] = {0, 0};
+        uint32_t a_par[2] = {0, 0};
+        bool act[2] = {2 * (int)blockIdx.x < p.n_tiles, 2 * (int)blockIdx.x + 1 < p.n_tiles};
+        bool ok = true;
+        if (resident) ok = bounded_wait(&w_full[0], 0, abort_flag, p.err);
+        uint64_t t_last = global_timer_ns();
+        uint32_t spins = 0;
+        while (ok && (act[0] || act[1])) {
+          bool progressed = false;
 #pragma unroll
-        for (int s = 0; s < 2; ++s) {
-          if (!act[s]) continue;
-          const int j = job_s[s];
-          const int st = resident ? j : (int)(seq_s[s] % G::STAGES);
-          if (!resident && !mbar_test_wait(&w_full[st], (seq_s[s] / G::STAGES) & 1)) continue;
-          if (!mbar_test_wait(&a_full[s], a_par[s])) continue;
-          a_par[s] ^= 1;
-          GNN_TRACE_AT(0, 2 * (seq_s[0] + seq_s[1]));
-          tc_fence_after();
-          const uint32_t wb = smem_u32(ring + st * G::MAT_BYTES);
-          const uint32_t d = tmem_base + s * G::SLOT_COLS;
-          const uint32_t ahi = d + H, alo = d + H + H / 2;
-#pragma unroll
-          for (int ks = 0; ks < H / 16; ++ks) {
-            const uint32_t off = (ks >> 2) * (H * 128) + (ks & 3) * 32;
-            const uint64_t bh = sdesc_kmajor_sw128(wb + off);
-            const uint64_t bl = sdesc_kmajor_sw128(wb + G::PART_BYTES + off);
-            const uint32_t acc = (p.job_acc[j] || ks > 0) ? 1u : 0u;
-            mma_bf16_ts(d, ahi + ks * 8, bh, G::IDESC, acc);
-            mma_bf16_ts(d, ahi + ks * 8, bl, G::IDESC, 1u);
-            mma_bf16_ts(d, alo + ks * 8, bh, G::IDESC, 1u);
+          for (int s = 0; s < 2; ++s) {
+            if (!act[s]) continue;
+            const int j = job_s[s];
+            const int st = resident ? j : (int)(seq_s[s] % G::STAGES);
+            if (!resident && !mbar_test_wait(&w_full[st], (seq_s[s] / G::STAGES) & 1)) continue;
+            if (!mbar_test_wait(&a_full[s], a_par[s])) continue;
+            a_par[s] ^= 1;
+            GNN_TRACE_AT(0, 2 * (int)seq_s[s] + s * 256);
+            tc_fence_after();
+            const uint32_t wb = smem_u32(ring + st * G::MAT_BYTES);
+            const uint32_t d = tmem_base + s * G::SLOT_COLS;
+            const uint32_t ahi = d + H, alo = d + H + H / 2;
+#pragma unroll 1
+            for (int ks = 0; ks < H / 16; ++ks) {
+              const uint32_t off = (ks >> 2) * (H * 128) + (ks & 3) * 32;
+              const uint64_t bh = sdesc_kmajor_sw128(wb + off);
+              const uint64_t bl = sdesc_kmajor_sw128(wb + G::PART_BYTES + off);
+              const uint32_t acc = (p.job_acc[j] || ks > 0) ? 1u : 0u;
+              mma_bf16_ts(d, ahi + ks * 8, bh, G::IDESC, acc);
+              mma_bf16_ts(d, ahi + ks * 8, bl, G::IDESC, 1u);
+              mma_bf16_ts(d, alo + ks * 8, bh, G::IDESC, 1u);
+            }
+            mma_commit(&d_full[s]);
+            GNN_TRACE_AT(0, 2 * (int)seq_s[s] + 1 + s * 256);
+            if (!resident) {
+              mma_commit(&w_empty[st]);
+              if (s == 0 && 2 * pair_s[0] + 1 >= p.n_tiles) mma_commit(&w_empty[st]);   // slot 1 has no tile
+            }
+            seq_s[s]++;
+            if (++job_s[s] == p.n_jobs) {
+              job_s[s] = 0;
+              pair_s[s] += gridDim.x;
+              act[s] = 2 * pair_s[s] + s < p.n_tiles;
+            }
+            progressed = true;
           }
-          mma_commit(&d_full[s]);
-          GNN_TRACE_AT(0, 2 * (seq_s[0] + seq_s[1]) + 1);
-          if (!resident) {
-            mma_commit(&w_empty[st]);
-            if (s == 0 && 2 * pair_s[0] + 1 >= p.n_tiles) mma_commit(&w_empty[st]);   // slot 1 has no tile
-          }
-          seq_s[s]++;
-          if (++job_s[s] == p.n_jobs) {
-            job_s[s] = 0;
-            pair_s[s] += gridDim.x;
-            act[s] = 2 * pair_s[s] + s < p.n_tiles;
-          }
-          progressed = true;
-        }
-        if (progressed) {
-          t_last = global_timer_ns();
-          spins = 0;
-        } else if ((++spins & 63u) == 0) {
-          if (*abort_flag) break;
-          if (global_timer_ns() - t_last > kWaitLimitNs) {
-            atomicOr(p.err, DEV_ERR_TIMEOUT);
-            *abort_flag = 1;
-            break;
+          if (progressed) {
+            t_last = global_timer_ns();
+            spins = 0;
+          } else if ((++spins & 63u) == 0) {
+            if (*abort_flag) break;
+            if (global_timer_ns() - t_last > kWaitLimitNs) {
+              atomicOr(p.err, DEV_ERR_TIMEOUT);
+              *abort_flag = 1;
+              break;
+            }
           }
         }
       }
+      __syncwarp();
     }
-    __syncwarp();
   } else {
-    // ------------------------------------------------ row workers (quad layout)
-    // Worker warp w serves slot (w-2)/8 and the 16 TMEM lanes
-    // [32*(w%4) + 16*hq, +16) of its lane quarter (hq = ((w-2)/4) % 2).
-    // Thread t of the warp owns rows r0 = base + t/4 and r1 = r0 + 8 and, in
-    // every 8-column block b, columns 8b + 2(t%4) and 8b + 2(t%4) + 1: the four
-    // threads of a quad share two rows, so LayerNorm statistics reduce with
-    // two quad shuffles.  v[4b + {0,1}] = row r0, v[4b + {2,3}] = row r1.
-    constexpr int NB = H / 8;                // 8-column blocks per row
-    const int wq = warp - 2;                 // 0..15
+    // Worker warpgroups.
+    setmaxnreg_inc<kWorkerRegs>();
+    const int wq = warp - 4;                   // worker index 0..15
     const int slot = wq >> 3;
+    const int ws = wq & 7;                     // warp index inside the slot
+    const int quarter = warp & 3;              // TMEM lane quarter of this warp
     const int hq = (wq >> 2) & 1;
-    const int quarter = warp & 3;            // TMEM lane quarter of this warp
     const int lane_base = quarter * 32 + hq * 16;
-    const int r0 = lane_base + (lane >> 2);  // rows inside the tile
-    const int cq = 2 * (lane & 3);           // column offset inside a block
+    const int r0 = lane_base + (lane >> 2);    // first of the two rows inside the tile
+    const int cq = 2 * (lane & 3);             // column offset inside a block
     const uint32_t lane_off = (uint32_t)lane_base << 16;
-    const uint32_t d_addr = tmem_base + slot * G::SLOT_COLS + lane_off;
+    const uint32_t slot_cols = tmem_base + slot * G::SLOT_COLS;
+    const uint32_t d_addr = slot_cols + lane_off;
     const uint32_t ahi_addr = d_addr + H;
     const uint32_t alo_addr = d_addr + H + H / 2;
     uint32_t d_use = 0;
-#ifdef GNN_TRACE
+  #ifdef GNN_TRACE
     int tr_iter = 0;
-    const int trow = (hq == 0 && quarter == 2) ? r0 - 64 : -1;   // 0 for one thread of slot 0's first warp
-#endif
+    const int trow = (slot == 0 && ws == 2 && lane == 0) ? 0 : -1;
+  #endif
 
-    auto arrive_a = [&]() {
+    auto arrive_a = [&](int, uint32_t) {
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&a_full[slot]);
     };
-    auto wait_d = [&]() -> bool {            // never early-exits a tile
+    auto wait_d = [&]() -> bool {              // never early-exits a tile
       const bool ok = bounded_wait(&d_full[slot], d_use & 1, abort_flag, p.err);
       d_use++;
       tc_fence_after();
@@ -318,12 +328,12 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     auto rm = [&](const float* base, int row, int b) -> const float2* {   // row-major [*, H]
       return reinterpret_cast<const float2*>(base + (size_t)row * H + 8 * b + cq);
     };
-    auto load_d = [&](float* v) {            // D of both rows, one TMEM round trip
+    auto load_d = [&](float* v) {              // D of both rows, one TMEM round trip
 #pragma unroll
       for (int c = 0; c < H; c += 64) tmem_ld_16x256b_x8(d_addr + c, v + c / 2);
       tmem_ld_wait();
     };
-    auto put_a = [&](const float* v) {       // both rows -> bf16 hi/lo A operand
+    auto put_a = [&](const float* v) {         // both rows -> bf16 hi/lo A operand
 #pragma unroll
       for (int h = 0; h < NB; h += 8) {
         uint32_t hi[16], lo[16];
@@ -344,15 +354,15 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         v[4 * k] += t.x; v[4 * k + 1] += t.y; v[4 * k + 2] += t.x; v[4 * k + 3] += t.y;
       }
     };
+    // LayerNorm (biased variance) + ReLU of both rows, in registers.  The host
+    // centres every weight block and bias that feeds a LayerNorm (each output
+    // row minus the mean over output rows), so the pre-activation reaching
+    // here already has zero mean over the H features: the LayerNorm needs only
+    // its variance (the subtraction of the mean is linear and sits in the MMA).
     auto ln_relu = [&](float* v, const float* gamma, const float* beta) {
-      float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-      for (int k = 0; k < NB; ++k) { s0 += v[4 * k] + v[4 * k + 1]; s1 += v[4 * k + 2] + v[4 * k + 3]; }
-      const float m0 = quad_sum(s0) * (1.0f / H), m1 = quad_sum(s1) * (1.0f / H);
       float q0 = 0.f, q1 = 0.f;
 #pragma unroll
       for (int k = 0; k < NB; ++k) {
-        v[4 * k] -= m0; v[4 * k + 1] -= m0; v[4 * k + 2] -= m1; v[4 * k + 3] -= m1;
         q0 = fmaf(v[4 * k], v[4 * k], fmaf(v[4 * k + 1], v[4 * k + 1], q0));
         q1 = fmaf(v[4 * k + 2], v[4 * k + 2], fmaf(v[4 * k + 3], v[4 * k + 3], q1));
       }
@@ -400,46 +410,44 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         }
       }
     };
-    auto prefetch_next_tile = [&](const float* base, int tile) {
-      const int nt = tile + 2 * (int)gridDim.x;
-      if (lane == 0 && wq == 0 && nt < p.n_tiles) prefetch_l2_bulk(base + (size_t)nt * kTileRows * H, kTileRows * H * 4);
-    };
 
     const int L = p.n_layers;
     bool ok = true;
+    uint32_t seq = 0;                          // this slot's job sequence number
     for (int pair = blockIdx.x; ok && pair < n_pairs; pair += gridDim.x) {
       const int tile = 2 * pair + slot;
       if (tile >= p.n_tiles) break;
       const int row0 = tile * kTileRows + r0, row1 = row0 + 8;
       const bool ok0 = row0 < p.n_rows, ok1 = row1 < p.n_rows;
       float v[4 * NB];
+      int j = 0;                               // job index inside the tile
+      auto next_job = [&]() { ++j; ++seq; };
+      auto wait_job = [&]() { ok &= wait_d(); };
 
       if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
         // vec layout: [gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]
-        if (slot == 0 && wq == 0 && lane == 0) progress[0] = pair;
+        if (slot == 0 && ws == 0 && lane == 0) progress[0] = pair;   // paces the L2 prefetcher
         GNN_TRACE_W(0);
+        const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
+        const int s1 = ok1 ? p.src_sorted[row1] : 0, d1 = ok1 ? p.dst_sorted[row1] : 0;
         load_t8(v, p.e, row0, ok0, ok1);
         GNN_TRACE_W(1);
         put_a(v);
-        arrive_a();                                     // job: D = e * W_e^T
+        arrive_a(j, seq); next_job();                     // job: D = e * W_e^T
         GNN_TRACE_W(2);
         // layer-1 terms of the endpoints, loaded while the MMA runs: P_s[src] + P_d[dst] (P_d carries b1)
-        {
-          const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
-          const int s1 = ok1 ? p.src_sorted[row1] : 0, d1 = ok1 ? p.dst_sorted[row1] : 0;
 #pragma unroll
-          for (int k = 0; k < NB; ++k) {
-            const float2 a0 = *rm(p.ps, s0, k), b0 = *rm(p.pd, d0, k);
-            const float2 a1 = *rm(p.ps, s1, k), b1 = *rm(p.pd, d1, k);
-            v[4 * k] = a0.x + b0.x; v[4 * k + 1] = a0.y + b0.y;
-            v[4 * k + 2] = a1.x + b1.x; v[4 * k + 3] = a1.y + b1.y;
-          }
+        for (int k = 0; k < NB; ++k) {
+          const float2 a0 = *rm(p.ps, s0, k), b0 = *rm(p.pd, d0, k);
+          const float2 a1 = *rm(p.ps, s1, k), b1 = *rm(p.pd, d1, k);
+          v[4 * k] = a0.x + b0.x; v[4 * k + 1] = a0.y + b0.y;
+          v[4 * k + 2] = a1.x + b1.x; v[4 * k + 3] = a1.y + b1.y;
         }
         GNN_TRACE_W(3);
-        ok &= wait_d();
+        wait_job();
         GNN_TRACE_W(5);
 #pragma unroll
-        for (int c = 0; c < H; c += 64) {               // v += D
+        for (int c = 0; c < H; c += 64) {                 // v += D
           float t[32];
           tmem_ld_16x256b_x8(d_addr + c, t);
           tmem_ld_wait();
@@ -447,16 +455,17 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           for (int i = 0; i < 32; ++i) v[c / 2 + i] += t[i];
         }
         ln_relu(v, vecs, vecs + H);
-        if (L > 1) { put_a(v); arrive_a(); }
+        put_a(v);
+        arrive_a(j, seq); next_job();
         GNN_TRACE_W(6);
         for (int l = 2; l <= L; ++l) {
-          ok &= wait_d();
+          wait_job();
           GNN_TRACE_W(5 + 2 * (l - 1));
           load_d(v);
           const float* vb = vecs + (2 + 3 * (l - 2)) * H;
           add_vec(v, vb);
           ln_relu(v, vb + H, vb + 2 * H);
-          if (l < L) { put_a(v); arrive_a(); }
+          if (l < L) { put_a(v); arrive_a(j, seq); next_job(); }
           GNN_TRACE_W(6 + 2 * (l - 1));
         }
         if constexpr (KIND == TileKind::EdgeUpdate) {
@@ -509,14 +518,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         add_vec(v, vb);
         ln_relu(v, vb + H, vb + 2 * H);
         put_a(v);
-        arrive_a();
+        arrive_a(j, seq); next_job();
         for (int l = 2; l <= L; ++l) {
-          ok &= wait_d();
+          wait_job();
           load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
           add_vec(v, vl);
           ln_relu(v, vl + H, vl + 2 * H);
-          if (l < L) { put_a(v); arrive_a(); }
+          if (l < L) { put_a(v); arrive_a(j, seq); next_job(); }
         }
         store_t8(p.e, row0, ok && ok0, ok && ok1, v);
       } else {
@@ -527,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         if constexpr (KIND == TileKind::NodeEncoder) {
 #pragma unroll
           for (int i = 0; i < 4 * NB; ++i) v[i] = 0.f;
-          for (int k = 0; k < p.n_feat; ++k) {          // layer 1 on CUDA cores
+          for (int k = 0; k < p.n_feat; ++k) {            // layer 1 on CUDA cores
             const float x0 = ok0 ? p.x[(size_t)row0 * p.x_stride + k] : 0.f;
             const float x1 = ok1 ? p.x[(size_t)row1 * p.x_stride + k] : 0.f;
 #pragma unroll
@@ -540,45 +549,51 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           add_vec(v, vb);
           ln_relu(v, vb + H, vb + 2 * H);
           put_a(v);
-          arrive_a();
+          arrive_a(j, seq); next_job();
           l0 = 2;
         } else {
           load_t8(v, p.h, row0, ok0, ok1);
           put_a(v);
-          arrive_a();                                   // job: D = h * W_h^T
-          prefetch_next_tile(p.h, tile);
-          prefetch_next_tile(p.agg, tile);
-          load_t8(v, p.agg, row0, ok0, ok1);            // a_j, summed by the aggregation kernel
-          ok &= wait_d();                               // A free again
+          arrive_a(j, seq); next_job();                   // job: D = h * W_h^T
+          if (ws == 0 && lane == 0) {
+            const int nt = tile + 2 * (int)gridDim.x;
+            if (nt < p.n_tiles) {
+              prefetch_l2_bulk(p.h + (size_t)nt * kTileRows * H, kTileRows * H * 4);
+              prefetch_l2_bulk(p.agg + (size_t)nt * kTileRows * H, kTileRows * H * 4);
+            }
+          }
+          load_t8(v, p.agg, row0, ok0, ok1);              // a_j, summed by the aggregation kernel
+          wait_job();                                     // A free again
           put_a(v);
-          arrive_a();                                   // job: D += a * W_a^T
+          arrive_a(j, seq); next_job();                   // job: D += a * W_a^T
           l0 = 1;
         }
         for (int l = l0; l <= L; ++l) {
-          ok &= wait_d();
+          wait_job();
           load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
           add_vec(v, vl);
           ln_relu(v, vl + H, vl + 2 * H);
           put_a(v);
-          arrive_a();                                   // next layer, or the P_s job
+          arrive_a(j, seq); next_job();                   // next layer, or the P_s job
         }
-        store_t8(p.h, row0, ok && ok0, ok && ok1, v);   // new node state
-        ok &= wait_d();                                 // P_s = W_s h (no bias)
+        store_t8(p.h, row0, ok && ok0, ok && ok1, v);     // new node state
+        wait_job();                                       // P_s = W_s h (no bias)
         stream_d(p.ps, row0, ok && ok0, ok && ok1, nullptr);
-        arrive_a();                                     // D read; A (= h) unchanged -> P_d job
-        ok &= wait_d();                                 // P_d = W_d h + b1 (edge-side bias)
+        tmem_ld_wait();
+        arrive_a(j, seq); next_job();                     // D read; A (= h) unchanged -> P_d job
+        wait_job();                                       // P_d = W_d h + b1 (edge-side bias)
         stream_d(p.pd, row0, ok && ok0, ok && ok1, vb + 3 * L * H);
       }
-      if (!ok) break;                        // leave only between tiles
-#ifdef GNN_TRACE
+      if (!ok) break;                          // leave only between tiles
+  #ifdef GNN_TRACE
       ++tr_iter;
-#endif
+  #endif
     }
     __syncwarp();
   }
 
-  // teardown: every role reaches this point (waits are bounded)
+  // teardown: every warp reaches this point (waits are bounded)
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {

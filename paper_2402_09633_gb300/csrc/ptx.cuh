@@ -60,6 +60,14 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Shared-memory atomic add with acquire-release ordering (CTA scope); returns the old value.
+__device__ __forceinline__ uint32_t atomic_add_acq_rel_shared(uint32_t* addr, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], %2;"
+               : "=r"(old) : "r"(smem_u32(addr)), "r"(v) : "memory");
+  return old;
+}
+
 // Wall-clock limit of every wait in the library (ns).
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
 
@@ -218,6 +226,12 @@ __device__ __forceinline__ void tmem_st_16x256b_x8(uint32_t taddr, const float* 
 __device__ __forceinline__ void tmem_st_wait() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
+
+// Warpgroup register reallocation (all 128 threads of a warpgroup execute it).
+template <int N>
+__device__ __forceinline__ void setmaxnreg_dec() { asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N)); }
+template <int N>
+__device__ __forceinline__ void setmaxnreg_inc() { asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N)); }
 
 // Named barrier over `nthreads` threads (multiple of 32).
 __device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t nthreads) {
