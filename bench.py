@@ -68,6 +68,38 @@ def step_model(w: S.Workload):
             "edge_update": edge_update, "node_update": node_update}
 
 
+# ------------------------------------------------------------------ ncu traffic
+PROFILE_FOR_KERNEL = {"edge_update": "edge_update_full_event.md"}
+KERNEL_SOURCES = ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh", "gnn_api.cu")
+
+
+def source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2402_09633_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary of `kernel`, or None when there is
+    none or the kernel sources changed since the counters were taken."""
+    name = PROFILE_FOR_KERNEL.get(kernel)
+    path = os.path.join(ROOT, "profiles", name) if name else None
+    if not path or not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            if ":" in line and line.split(":", 1)[0].strip() in ("source_sha256", "dram_bytes_per_launch"):
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.split()[0]
+    if fields.get("source_sha256") != source_hash() or "dram_bytes_per_launch" not in fields:
+        return None
+    return int(fields["dram_bytes_per_launch"])
+
+
 # ------------------------------------------------------------------ clocks
 def gpu_index_for(local_rank: int) -> str:
     vis = os.environ.get("CUDA_VISIBLE_DEVICES")
@@ -287,7 +319,7 @@ def run_gb300(args, rank: int, world: int, local: int):
     if dom_model is not None:
         achieved = dom_model["bytes"] / dom_avg_s / 1e9
         roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"],
-                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": profiled_traffic(dom),
                     "peak_source": f"{peak_src} (hbm_gbs, copy burst) -- of {peak_src}",
                     "bytes_per_launch": dom_model["bytes"], "avg_launch_ms": dom_avg_s * 1e3,
                     "tensor_tflops_executed": 3 * dom_model["flops"] / dom_avg_s / 1e12}

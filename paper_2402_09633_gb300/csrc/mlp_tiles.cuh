@@ -603,38 +603,48 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 }
 
 // a_j = sum of the messages m_ij of the edges into node j (CSR segment of j,
-// fixed slot order, no atomics).  One thread per (node, 8-column block): a
-// warp covers 32 consecutive nodes and one block, so both its loads (rows of
-// neighbouring segments, 32 bytes each) and its stores are contiguous.
+// no atomics).  A quad of lanes serves one (node, 8-column block): lane q sums
+// the segment rows q, q+4, q+8, ... in order, and the four partial sums are
+// combined by a fixed shuffle tree.  The order of additions therefore depends
+// only on the node's own segment (deterministic, and identical for a node
+// whether its event is scored alone or in a batch).  A quad reads 4
+// consecutive rows (128 contiguous bytes of the row-tiled state) per step.
 template <int H>
 __global__ void __launch_bounds__(256) aggregate_kernel(const float* __restrict__ e, const int* __restrict__ rowptr,
                                                         int n_nodes, float* __restrict__ agg) {
   constexpr int NB = H / 8;
-  const int b = blockIdx.y * 8 + (threadIdx.x >> 5);
-  const int j = blockIdx.x * 32 + (threadIdx.x & 31);
-  if (j >= n_nodes || b >= NB) return;
-  const int k0 = rowptr[j], k1 = rowptr[j + 1];
+  const int b = blockIdx.y;                          // 8-column block
+  const int q = threadIdx.x & 3;
+  const int j = blockIdx.x * 64 + (threadIdx.x >> 2);
+  const bool has = j < n_nodes;
+  const int k0 = has ? rowptr[j] : 0, k1 = has ? rowptr[j + 1] : 0;
   auto row = [&](int k) { return reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NB + b) * 128 + (k & 127)) * 8); };
   float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0;
-  int k = k0;
-  for (; k + 4 <= k1; k += 4) {              // four rows in flight, summed in slot order
-    float4 x[4], y[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) { x[u] = row(k + u)[0]; y[u] = row(k + u)[1]; }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      a0.x += x[u].x; a0.y += x[u].y; a0.z += x[u].z; a0.w += x[u].w;
-      a1.x += y[u].x; a1.y += y[u].y; a1.z += y[u].z; a1.w += y[u].w;
-    }
+  int k = k0 + q;
+  for (; k + 4 < k1; k += 8) {                       // two rows of this lane in flight
+    const float4 x0 = row(k)[0], y0 = row(k)[1], x1 = row(k + 4)[0], y1 = row(k + 4)[1];
+    a0.x += x0.x; a0.y += x0.y; a0.z += x0.z; a0.w += x0.w;
+    a1.x += y0.x; a1.y += y0.y; a1.z += y0.z; a1.w += y0.w;
+    a0.x += x1.x; a0.y += x1.y; a0.z += x1.z; a0.w += x1.w;
+    a1.x += y1.x; a1.y += y1.y; a1.z += y1.z; a1.w += y1.w;
   }
-  for (; k < k1; ++k) {
+  if (k < k1) {
     const float4 x = row(k)[0], y = row(k)[1];
     a0.x += x.x; a0.y += x.y; a0.z += x.z; a0.w += x.w;
     a1.x += y.x; a1.y += y.y; a1.z += y.z; a1.w += y.w;
   }
-  float4* o = reinterpret_cast<float4*>(agg + (((size_t)(j >> 7) * NB + b) * 128 + (j & 127)) * 8);
-  o[0] = a0;
-  o[1] = a1;
+#pragma unroll
+  for (int m = 1; m <= 2; m <<= 1) {
+    a0.x += __shfl_xor_sync(0xffffffffu, a0.x, m); a0.y += __shfl_xor_sync(0xffffffffu, a0.y, m);
+    a0.z += __shfl_xor_sync(0xffffffffu, a0.z, m); a0.w += __shfl_xor_sync(0xffffffffu, a0.w, m);
+    a1.x += __shfl_xor_sync(0xffffffffu, a1.x, m); a1.y += __shfl_xor_sync(0xffffffffu, a1.y, m);
+    a1.z += __shfl_xor_sync(0xffffffffu, a1.z, m); a1.w += __shfl_xor_sync(0xffffffffu, a1.w, m);
+  }
+  if (has && q == 0) {
+    float4* o = reinterpret_cast<float4*>(agg + (((size_t)(j >> 7) * NB + b) * 128 + (j & 127)) * 8);
+    o[0] = a0;
+    o[1] = a1;
+  }
 }
 
 }  // namespace gnn
