@@ -166,7 +166,8 @@ const char* gnn_error_string(int code);
  * input edge id), 2 src_sorted int32 [E], 3 node state h, 4 edge state e (CSR
  * order).  The states are float32 in the row-tiled layout of the kernels:
  * R = rows rounded up to a multiple of 128, element (r, c) at index
- * ((r / 128) * (H / 8) + c / 8) * 1024 + (r % 128) * 8 + c % 8, R * H floats.
+ * ((r / 128) * (H / 16) + bp) * 2048 + (r % 128) * 16 + x, R * H floats, where
+ * b = c / 8, bp = b / 2 and x = 4 * ((c % 8) / 2) + 2 * (b % 2) + c % 2.
  * Errors: INVALID_ARG when the buffer is unknown or `bytes` is too small.
  */
 int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_t stream);

@@ -321,12 +321,23 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
       x += __shfl_xor_sync(0xffffffffu, x, 2);
       return x;
     };
-    // Row-tiled state "T8": element (r, c) at ((r/128)*(H/8) + c/8)*1024 + (r%128)*8 + c%8.
-    auto t8 = [&](const float* base, int row, int b) -> const float2* {
-      return reinterpret_cast<const float2*>(base + (((size_t)(row >> 7) * NB + b) * 128 + (row & 127)) * 8 + cq);
+    // Row data keep each thread's four values of a block pair (blocks 2bp and 2bp+1, columns
+    // 2(t%4) and 2(t%4)+1 of each) together, so every row access is one 16-byte vector:
+    //   row-tiled state "T16" (e, h, a): (r, c) at ((r/128)*(H/16) + bp)*2048 + (r%128)*16 + x,
+    //   row-major "RM16" (P_s, P_d):     (r, c) at r*H + bp*16 + x,
+    // with b = c/8, bp = b/2, x = 4*((c%8)/2) + 2*(b%2) + c%2.
+    auto t16 = [&](const float* base, int row, int bp) -> const float4* {
+      return reinterpret_cast<const float4*>(base + (((size_t)(row >> 7) * (NB / 2) + bp) * 128 + (row & 127)) * 16 + 2 * cq);
     };
-    auto rm = [&](const float* base, int row, int b) -> const float2* {   // row-major [*, H]
-      return reinterpret_cast<const float2*>(base + (size_t)row * H + 8 * b + cq);
+    auto rm16 = [&](const float* base, int row, int bp) -> const float4* {
+      return reinterpret_cast<const float4*>(base + (size_t)row * H + bp * 16 + 2 * cq);
+    };
+    // (row r0 quad values of blocks 2bp, 2bp+1) <-> v
+    auto put4 = [&](float* v, int bp, int r, const float4& x) {
+      v[8 * bp + 2 * r] = x.x; v[8 * bp + 2 * r + 1] = x.y; v[8 * bp + 4 + 2 * r] = x.z; v[8 * bp + 4 + 2 * r + 1] = x.w;
+    };
+    auto get4 = [&](const float* v, int bp, int r) {
+      return make_float4(v[8 * bp + 2 * r], v[8 * bp + 2 * r + 1], v[8 * bp + 4 + 2 * r], v[8 * bp + 4 + 2 * r + 1]);
     };
     auto load_d = [&](float* v) {              // D of both rows, one TMEM round trip
 #pragma unroll
@@ -378,19 +389,19 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         v[4 * k + 3] = fmaxf(fmaf(v[4 * k + 3] * i1, g.y, b.y), 0.f);
       }
     };
-    auto load_t8 = [&](float* v, const float* base, int row0, bool ok0, bool ok1) {
+    auto load_t16 = [&](float* v, const float* base, int row0, bool ok0, bool ok1) {
+      const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int k = 0; k < NB; ++k) {
-        const float2 a = ok0 ? *t8(base, row0, k) : make_float2(0.f, 0.f);
-        const float2 b = ok1 ? *t8(base, row0 + 8, k) : make_float2(0.f, 0.f);
-        v[4 * k] = a.x; v[4 * k + 1] = a.y; v[4 * k + 2] = b.x; v[4 * k + 3] = b.y;
+      for (int bp = 0; bp < NB / 2; ++bp) {
+        put4(v, bp, 0, ok0 ? *t16(base, row0, bp) : z);
+        put4(v, bp, 1, ok1 ? *t16(base, row0 + 8, bp) : z);
       }
     };
-    auto store_t8 = [&](float* base, int row0, bool ok0, bool ok1, const float* v) {
+    auto store_t16 = [&](float* base, int row0, bool ok0, bool ok1, const float* v) {
 #pragma unroll
-      for (int k = 0; k < NB; ++k) {
-        if (ok0) *const_cast<float2*>(t8(base, row0, k)) = make_float2(v[4 * k], v[4 * k + 1]);
-        if (ok1) *const_cast<float2*>(t8(base, row0 + 8, k)) = make_float2(v[4 * k + 2], v[4 * k + 3]);
+      for (int bp = 0; bp < NB / 2; ++bp) {
+        if (ok0) *const_cast<float4*>(t16(base, row0, bp)) = get4(v, bp, 0);
+        if (ok1) *const_cast<float4*>(t16(base, row0 + 8, bp)) = get4(v, bp, 1);
       }
     };
     // D (+ bias) of both rows streamed to a row-major output, 8 blocks per TMEM round trip.
@@ -400,13 +411,18 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         float t[32];
         tmem_ld_16x256b_x8(d_addr + c, t);
         tmem_ld_wait();
+        if (bias) {
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const int kb = c / 8 + k;
-          float2 bb = make_float2(0.f, 0.f);
-          if (bias) bb = *reinterpret_cast<const float2*>(bias + 8 * kb + cq);
-          if (ok0) *const_cast<float2*>(rm(base, row0, kb)) = make_float2(t[4 * k] + bb.x, t[4 * k + 1] + bb.y);
-          if (ok1) *const_cast<float2*>(rm(base, row0 + 8, kb)) = make_float2(t[4 * k + 2] + bb.x, t[4 * k + 3] + bb.y);
+          for (int k = 0; k < 8; ++k) {
+            const float2 bb = *reinterpret_cast<const float2*>(bias + c + 8 * k + cq);
+            t[4 * k] += bb.x; t[4 * k + 1] += bb.y; t[4 * k + 2] += bb.x; t[4 * k + 3] += bb.y;
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {                    // block pairs of this 64-column chunk
+          const int bp = c / 16 + k;
+          if (ok0) *const_cast<float4*>(rm16(base, row0, bp)) = get4(t, k, 0);
+          if (ok1) *const_cast<float4*>(rm16(base, row0 + 8, bp)) = get4(t, k, 1);
         }
       }
     };
@@ -430,18 +446,18 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         GNN_TRACE_W(0);
         const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
         const int s1 = ok1 ? p.src_sorted[row1] : 0, d1 = ok1 ? p.dst_sorted[row1] : 0;
-        load_t8(v, p.e, row0, ok0, ok1);
+        load_t16(v, p.e, row0, ok0, ok1);
         GNN_TRACE_W(1);
         put_a(v);
         arrive_a(j, seq); next_job();                     // job: D = e * W_e^T
         GNN_TRACE_W(2);
         // layer-1 terms of the endpoints, loaded while the MMA runs: P_s[src] + P_d[dst] (P_d carries b1)
 #pragma unroll
-        for (int k = 0; k < NB; ++k) {
-          const float2 a0 = *rm(p.ps, s0, k), b0 = *rm(p.pd, d0, k);
-          const float2 a1 = *rm(p.ps, s1, k), b1 = *rm(p.pd, d1, k);
-          v[4 * k] = a0.x + b0.x; v[4 * k + 1] = a0.y + b0.y;
-          v[4 * k + 2] = a1.x + b1.x; v[4 * k + 3] = a1.y + b1.y;
+        for (int bp = 0; bp < NB / 2; ++bp) {
+          const float4 a0 = *rm16(p.ps, s0, bp), b0 = *rm16(p.pd, d0, bp);
+          const float4 a1 = *rm16(p.ps, s1, bp), b1 = *rm16(p.pd, d1, bp);
+          put4(v, bp, 0, make_float4(a0.x + b0.x, a0.y + b0.y, a0.z + b0.z, a0.w + b0.w));
+          put4(v, bp, 1, make_float4(a1.x + b1.x, a1.y + b1.y, a1.z + b1.z, a1.w + b1.w));
         }
         GNN_TRACE_W(3);
         wait_job();
@@ -469,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           GNN_TRACE_W(6 + 2 * (l - 1));
         }
         if constexpr (KIND == TileKind::EdgeUpdate) {
-          store_t8(p.e, row0, ok && ok0, ok && ok1, v);
+          store_t16(p.e, row0, ok && ok0, ok && ok1, v);
           GNN_TRACE_W(11);
         } else {
           const float* wo = vecs + (2 + 3 * (L - 1)) * H;
@@ -527,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           ln_relu(v, vl + H, vl + 2 * H);
           if (l < L) { put_a(v); arrive_a(j, seq); next_job(); }
         }
-        store_t8(p.e, row0, ok && ok0, ok && ok1, v);
+        store_t16(p.e, row0, ok && ok0, ok && ok1, v);
       } else {
         // NodeEncoder / NodeUpdate.
         // vec layout: [W1^T (n_feat x H) if encoder], (b_l, gamma_l, beta_l) for l = 1..L, b1_edge
@@ -552,9 +568,11 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           arrive_a(j, seq); next_job();
           l0 = 2;
         } else {
-          load_t8(v, p.h, row0, ok0, ok1);
+          GNN_TRACE_W(0);
+          load_t16(v, p.h, row0, ok0, ok1);
           put_a(v);
           arrive_a(j, seq); next_job();                   // job: D = h * W_h^T
+          GNN_TRACE_W(1);
           if (ws == 0 && lane == 0) {
             const int nt = tile + 2 * (int)gridDim.x;
             if (nt < p.n_tiles) {
@@ -562,28 +580,38 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
               prefetch_l2_bulk(p.agg + (size_t)nt * kTileRows * H, kTileRows * H * 4);
             }
           }
-          load_t8(v, p.agg, row0, ok0, ok1);              // a_j, summed by the aggregation kernel
+          load_t16(v, p.agg, row0, ok0, ok1);              // a_j, summed by the aggregation kernel
+          GNN_TRACE_W(2);
           wait_job();                                     // A free again
+          GNN_TRACE_W(3);
           put_a(v);
           arrive_a(j, seq); next_job();                   // job: D += a * W_a^T
+          GNN_TRACE_W(4);
           l0 = 1;
         }
         for (int l = l0; l <= L; ++l) {
           wait_job();
+          GNN_TRACE_W(3 + 2 * l);
           load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
           add_vec(v, vl);
           ln_relu(v, vl + H, vl + 2 * H);
           put_a(v);
           arrive_a(j, seq); next_job();                   // next layer, or the P_s job
+          GNN_TRACE_W(4 + 2 * l);
         }
-        store_t8(p.h, row0, ok && ok0, ok && ok1, v);     // new node state
+        store_t16(p.h, row0, ok && ok0, ok && ok1, v);     // new node state
+        GNN_TRACE_W(11);
         wait_job();                                       // P_s = W_s h (no bias)
+        GNN_TRACE_W(12);
         stream_d(p.ps, row0, ok && ok0, ok && ok1, nullptr);
         tmem_ld_wait();
         arrive_a(j, seq); next_job();                     // D read; A (= h) unchanged -> P_d job
+        GNN_TRACE_W(13);
         wait_job();                                       // P_d = W_d h + b1 (edge-side bias)
+        GNN_TRACE_W(14);
         stream_d(p.pd, row0, ok && ok0, ok && ok1, vb + 3 * L * H);
+        GNN_TRACE_W(15);
       }
       if (!ok) break;                          // leave only between tiles
   #ifdef GNN_TRACE
@@ -603,48 +631,35 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 }
 
 // a_j = sum of the messages m_ij of the edges into node j (CSR segment of j,
-// no atomics).  A quad of lanes serves one (node, 8-column block): lane q sums
-// the segment rows q, q+4, q+8, ... in order, and the four partial sums are
-// combined by a fixed shuffle tree.  The order of additions therefore depends
-// only on the node's own segment (deterministic, and identical for a node
-// whether its event is scored alone or in a batch).  A quad reads 4
-// consecutive rows (128 contiguous bytes of the row-tiled state) per step.
+// summed in slot order, no atomics: deterministic, and identical for a node
+// whether its event is scored alone or in a batch).  A quad of lanes serves
+// one (node, 16-column block pair); lane q owns one 16-byte vector of the
+// pair's 64-byte piece of a row (row-tiled T16 layout of the tile kernels),
+// so a quad reads 64 contiguous bytes per row, four rows in flight.
 template <int H>
 __global__ void __launch_bounds__(256) aggregate_kernel(const float* __restrict__ e, const int* __restrict__ rowptr,
                                                         int n_nodes, float* __restrict__ agg) {
-  constexpr int NB = H / 8;
-  const int b = blockIdx.y;                          // 8-column block
+  constexpr int NBP = H / 16;
+  const int bp = blockIdx.y;                         // block pair
   const int q = threadIdx.x & 3;
   const int j = blockIdx.x * 64 + (threadIdx.x >> 2);
-  const bool has = j < n_nodes;
-  const int k0 = has ? rowptr[j] : 0, k1 = has ? rowptr[j + 1] : 0;
-  auto row = [&](int k) { return reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NB + b) * 128 + (k & 127)) * 8); };
-  float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0;
-  int k = k0 + q;
-  for (; k + 4 < k1; k += 8) {                       // two rows of this lane in flight
-    const float4 x0 = row(k)[0], y0 = row(k)[1], x1 = row(k + 4)[0], y1 = row(k + 4)[1];
-    a0.x += x0.x; a0.y += x0.y; a0.z += x0.z; a0.w += x0.w;
-    a1.x += y0.x; a1.y += y0.y; a1.z += y0.z; a1.w += y0.w;
-    a0.x += x1.x; a0.y += x1.y; a0.z += x1.z; a0.w += x1.w;
-    a1.x += y1.x; a1.y += y1.y; a1.z += y1.z; a1.w += y1.w;
+  if (j >= n_nodes) return;
+  const int k0 = rowptr[j], k1 = rowptr[j + 1];
+  auto at = [&](int k) { return *reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NBP + bp) * 128 + (k & 127)) * 16 + 4 * q); };
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+  int k = k0;
+  for (; k + 4 <= k1; k += 4) {
+    const float4 x0 = at(k), x1 = at(k + 1), x2 = at(k + 2), x3 = at(k + 3);
+    a.x += x0.x; a.y += x0.y; a.z += x0.z; a.w += x0.w;
+    a.x += x1.x; a.y += x1.y; a.z += x1.z; a.w += x1.w;
+    a.x += x2.x; a.y += x2.y; a.z += x2.z; a.w += x2.w;
+    a.x += x3.x; a.y += x3.y; a.z += x3.z; a.w += x3.w;
   }
-  if (k < k1) {
-    const float4 x = row(k)[0], y = row(k)[1];
-    a0.x += x.x; a0.y += x.y; a0.z += x.z; a0.w += x.w;
-    a1.x += y.x; a1.y += y.y; a1.z += y.z; a1.w += y.w;
+  for (; k < k1; ++k) {
+    const float4 x = at(k);
+    a.x += x.x; a.y += x.y; a.z += x.z; a.w += x.w;
   }
-#pragma unroll
-  for (int m = 1; m <= 2; m <<= 1) {
-    a0.x += __shfl_xor_sync(0xffffffffu, a0.x, m); a0.y += __shfl_xor_sync(0xffffffffu, a0.y, m);
-    a0.z += __shfl_xor_sync(0xffffffffu, a0.z, m); a0.w += __shfl_xor_sync(0xffffffffu, a0.w, m);
-    a1.x += __shfl_xor_sync(0xffffffffu, a1.x, m); a1.y += __shfl_xor_sync(0xffffffffu, a1.y, m);
-    a1.z += __shfl_xor_sync(0xffffffffu, a1.z, m); a1.w += __shfl_xor_sync(0xffffffffu, a1.w, m);
-  }
-  if (has && q == 0) {
-    float4* o = reinterpret_cast<float4*>(agg + (((size_t)(j >> 7) * NB + b) * 128 + (j & 127)) * 8);
-    o[0] = a0;
-    o[1] = a1;
-  }
+  *reinterpret_cast<float4*>(agg + (((size_t)(j >> 7) * NBP + bp) * 128 + (j & 127)) * 16 + 4 * q) = a;
 }
 
 }  // namespace gnn

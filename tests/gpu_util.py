@@ -43,7 +43,11 @@ def check_parity(s_gpu, W, x, ei, T, tol=LOGIT_TOL_FP32, eps=1e-5):
 
 
 def untile(buf, n_rows, H):
-    """Row-tiled state [R/128][H/8][128][8] -> row-major [n_rows, H]."""
+    """Row-tiled state (T16 layout, see gnn_debug_copy in include/gnn.h) -> row-major [n_rows, H]."""
     R = (n_rows + 127) // 128 * 128
-    a = np.asarray(buf).reshape(R // 128, H // 8, 128, 8).transpose(0, 2, 1, 3).reshape(R, H)
-    return a[:n_rows]
+    c = np.arange(H)
+    b = c // 8
+    x = 4 * ((c % 8) // 2) + 2 * (b % 2) + c % 2
+    r = np.arange(R)
+    idx = (((r[:, None] // 128) * (H // 16) + (b // 2)[None, :]) * 2048 + (r[:, None] % 128) * 16 + x[None, :])
+    return np.asarray(buf)[idx][:n_rows]
