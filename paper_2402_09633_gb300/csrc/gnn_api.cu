@@ -209,8 +209,8 @@ int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStr
     launch_tile<TileKind::EdgeUpdate, H>(c, c->plan[3], pe, st);
     {
       const int pr = prof_begin(c, 7, 1, st);
-      const dim3 grid((N + 63) / 64, H / 16);
-      aggregate_kernel<H><<<grid, 256, 0, st>>>(c->e, c->rowptr, N, c->agg);
+      constexpr int npb = agg_nodes_per_block<H>();
+      aggregate_kernel<H><<<(N + npb - 1) / npb, 256, 0, st>>>(c->e, c->rowptr, N, c->agg);
       prof_end(c, pr, st);
     }
     launch_tile<TileKind::NodeUpdate, H>(c, c->plan[t < T ? 4 : 5], pn, st);

@@ -631,21 +631,26 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 }
 
 // a_j = sum of the messages m_ij of the edges into node j (CSR segment of j,
-// summed in slot order, no atomics: deterministic, and identical for a node
-// whether its event is scored alone or in a batch).  A quad of lanes serves
-// one (node, 16-column block pair); lane q owns one 16-byte vector of the
-// pair's 64-byte piece of a row (row-tiled T16 layout of the tile kernels),
-// so a quad reads 64 contiguous bytes per row, four rows in flight.
+// summed in slot order from zero, no atomics: deterministic, and identical for
+// a node whether its event is scored alone or in a batch).  One warp serves one
+// node (half a warp when H = 64): lane 4*bp + q owns the 16-byte vector q of
+// block pair bp (row-tiled T16 layout of the tile kernels), so all lanes of a
+// node run the same number of steps whatever the degree distribution, and
+// every message row is read in whole 64-byte pieces.
+template <int H>
+constexpr int agg_nodes_per_block() { return 256 / (H / 4); }
+
 template <int H>
 __global__ void __launch_bounds__(256) aggregate_kernel(const float* __restrict__ e, const int* __restrict__ rowptr,
                                                         int n_nodes, float* __restrict__ agg) {
   constexpr int NBP = H / 16;
-  const int bp = blockIdx.y;                         // block pair
-  const int q = threadIdx.x & 3;
-  const int j = blockIdx.x * 64 + (threadIdx.x >> 2);
+  constexpr int LPN = H / 4;                         // lanes per node
+  const int li = threadIdx.x % LPN;
+  const int bp = li >> 2, q = li & 3;
+  const int j = blockIdx.x * agg_nodes_per_block<H>() + (int)threadIdx.x / LPN;
   if (j >= n_nodes) return;
   const int k0 = rowptr[j], k1 = rowptr[j + 1];
-  auto at = [&](int k) { return *reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NBP + bp) * 128 + (k & 127)) * 16 + 4 * q); };
+  auto at = [&](int k) { return __ldcs(reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NBP + bp) * 128 + (k & 127)) * 16 + 4 * q)); };
   float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
   int k = k0;
   for (; k + 4 <= k1; k += 4) {
