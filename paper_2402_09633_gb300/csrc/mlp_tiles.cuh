@@ -344,17 +344,36 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
       for (int c = 0; c < H; c += 64) tmem_ld_16x256b_x8(d_addr + c, v + c / 2);
       tmem_ld_wait();
     };
-    auto put_a = [&](const float* v) {         // both rows -> bf16 hi/lo A operand
+    // Blocks 4k..4k+3 of both rows (t[4b..4b+3] = block 4k+b: row 0 cols 2(t%4), +1; row 1 the same)
+    // -> bf16 hi/lo A operand.  No wait: the caller ends a run of stores with tmem_st_wait().
+    auto put_a_chunk = [&](int k, const float* t) {
+      uint32_t hi[8], lo[8];
 #pragma unroll
-      for (int h = 0; h < NB; h += 8) {
-        uint32_t hi[16], lo[16];
+      for (int b = 0; b < 4; ++b) {
+        split_bf16x2(t[4 * b], t[4 * b + 1], hi[2 * b], lo[2 * b]);
+        split_bf16x2(t[4 * b + 2], t[4 * b + 3], hi[2 * b + 1], lo[2 * b + 1]);
+      }
+      tmem_st_16x128b_x4(ahi_addr + 16 * k, hi);
+      tmem_st_16x128b_x4(alo_addr + 16 * k, lo);
+    };
+    // both rows -> bf16 hi/lo A operand (8 blocks per store in the edge kernels, whose
+    // epilogues keep whole rows in registers; 4 in the others, which stream)
+    auto put_a = [&](const float* v) {
+      if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
 #pragma unroll
-        for (int b = 0; b < 8; ++b) {
-          split_bf16x2(v[4 * (h + b)], v[4 * (h + b) + 1], hi[2 * b], lo[2 * b]);
-          split_bf16x2(v[4 * (h + b) + 2], v[4 * (h + b) + 3], hi[2 * b + 1], lo[2 * b + 1]);
+        for (int h = 0; h < NB; h += 8) {
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int b = 0; b < 8; ++b) {
+            split_bf16x2(v[4 * (h + b)], v[4 * (h + b) + 1], hi[2 * b], lo[2 * b]);
+            split_bf16x2(v[4 * (h + b) + 2], v[4 * (h + b) + 3], hi[2 * b + 1], lo[2 * b + 1]);
+          }
+          tmem_st_16x128b_x8(ahi_addr + 4 * h, hi);
+          tmem_st_16x128b_x8(alo_addr + 4 * h, lo);
         }
-        tmem_st_16x128b_x8(ahi_addr + 4 * h, hi);
-        tmem_st_16x128b_x8(alo_addr + 4 * h, lo);
+      } else {
+#pragma unroll
+        for (int k = 0; k < NB / 4; ++k) put_a_chunk(k, v + 16 * k);
       }
       tmem_st_wait();
     };
@@ -389,6 +408,59 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         v[4 * k + 3] = fmaxf(fmaf(v[4 * k + 3] * i1, g.y, b.y), 0.f);
       }
     };
+    // LayerNorm + ReLU of D + bias of both rows, streamed from tensor memory in
+    // two passes (the squares for the variance, then the values), so that a
+    // thread holds at most 32 columns at a time; emit(k, t) receives blocks
+    // 4k..4k+3 in the put_a_chunk order.  D stays valid until the slot's next
+    // MMA, which this thread has not released yet.
+    auto ln_stream = [&](const float* bias, const float* gamma, const float* beta, auto&& emit) {
+      float q0 = 0.f, q1 = 0.f;
+      {
+        float t[H / 2];
+#pragma unroll
+        for (int c = 0; c < H; c += 64) tmem_ld_16x256b_x8(d_addr + c, t + c / 2);
+        tmem_ld_wait();
+#pragma unroll
+        for (int k = 0; k < NB; ++k) {
+          const float2 bb = *reinterpret_cast<const float2*>(bias + 8 * k + cq);
+          const float a0 = t[4 * k] + bb.x, a1 = t[4 * k + 1] + bb.y;
+          const float c0 = t[4 * k + 2] + bb.x, c1 = t[4 * k + 3] + bb.y;
+          q0 = fmaf(a0, a0, fmaf(a1, a1, q0));
+          q1 = fmaf(c0, c0, fmaf(c1, c1, q1));
+        }
+      }
+      const float i0 = rsqrtf(quad_sum(q0) * (1.0f / H) + p.eps);
+      const float i1 = rsqrtf(quad_sum(q1) * (1.0f / H) + p.eps);
+      float t[2][16];                          // double buffer: chunk k+1 is read while chunk k is emitted
+      tmem_ld_16x256b_x4(d_addr, t[0]);
+      tmem_ld_wait();
+#pragma unroll
+      for (int k = 0; k < NB / 4; ++k) {
+        if (k + 1 < NB / 4) tmem_ld_16x256b_x4(d_addr + 32 * (k + 1), t[(k + 1) & 1]);
+        float* u = t[k & 1];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          const int col = 32 * k + 8 * b + cq;
+          const float2 bb = *reinterpret_cast<const float2*>(bias + col);
+          const float2 g = *reinterpret_cast<const float2*>(gamma + col);
+          const float2 be = *reinterpret_cast<const float2*>(beta + col);
+          u[4 * b] = fmaxf(fmaf((u[4 * b] + bb.x) * i0, g.x, be.x), 0.f);
+          u[4 * b + 1] = fmaxf(fmaf((u[4 * b + 1] + bb.y) * i0, g.y, be.y), 0.f);
+          u[4 * b + 2] = fmaxf(fmaf((u[4 * b + 2] + bb.x) * i1, g.x, be.x), 0.f);
+          u[4 * b + 3] = fmaxf(fmaf((u[4 * b + 3] + bb.y) * i1, g.y, be.y), 0.f);
+        }
+        emit(k, u);
+        if (k + 1 < NB / 4) tmem_ld_wait();
+      }
+    };
+    // blocks 4k..4k+3 of both rows -> row-tiled (T16) output rows
+    auto store_t16_chunk = [&](float* base, int row0, bool ok0, bool ok1, int k, const float* t) {
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        if (ok0) *const_cast<float4*>(t16(base, row0, 2 * k + j)) = get4(t, j, 0);
+        if (ok1) *const_cast<float4*>(t16(base, row0 + 8, 2 * k + j)) = get4(t, j, 1);
+      }
+    };
     auto load_t16 = [&](float* v, const float* base, int row0, bool ok0, bool ok1) {
       const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -404,22 +476,22 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         if (ok1) *const_cast<float4*>(t16(base, row0 + 8, bp)) = get4(v, bp, 1);
       }
     };
-    // D (+ bias) of both rows streamed to a row-major output, 8 blocks per TMEM round trip.
+    // D (+ bias) of both rows streamed to a row-major output, 4 blocks per TMEM round trip.
     auto stream_d = [&](float* base, int row0, bool ok0, bool ok1, const float* bias) {
 #pragma unroll
-      for (int c = 0; c < H; c += 64) {
-        float t[32];
-        tmem_ld_16x256b_x8(d_addr + c, t);
+      for (int c = 0; c < H; c += 32) {
+        float t[16];
+        tmem_ld_16x256b_x4(d_addr + c, t);
         tmem_ld_wait();
         if (bias) {
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
+          for (int k = 0; k < 4; ++k) {
             const float2 bb = *reinterpret_cast<const float2*>(bias + c + 8 * k + cq);
             t[4 * k] += bb.x; t[4 * k + 1] += bb.y; t[4 * k + 2] += bb.x; t[4 * k + 3] += bb.y;
           }
         }
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {                    // block pairs of this 64-column chunk
+        for (int k = 0; k < 2; ++k) {                    // block pairs of this 32-column chunk
           const int bp = c / 16 + k;
           if (ok0) *const_cast<float4*>(rm16(base, row0, bp)) = get4(t, k, 0);
           if (ok1) *const_cast<float4*>(rm16(base, row0 + 8, bp)) = get4(t, k, 1);
@@ -535,15 +607,19 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         ln_relu(v, vb + H, vb + 2 * H);
         put_a(v);
         arrive_a(j, seq); next_job();
-        for (int l = 2; l <= L; ++l) {
+        for (int l = 2; l < L; ++l) {
           wait_job();
-          load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
-          add_vec(v, vl);
-          ln_relu(v, vl + H, vl + 2 * H);
-          if (l < L) { put_a(v); arrive_a(j, seq); next_job(); }
+          ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { put_a_chunk(k, t); });
+          tmem_st_wait();
+          arrive_a(j, seq); next_job();
         }
-        store_t16(p.e, row0, ok && ok0, ok && ok1, v);
+        wait_job();
+        {
+          const float* vl = vb + 3 * (L - 1) * H;
+          const bool w0 = ok && ok0, w1 = ok && ok1;
+          ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { store_t16_chunk(p.e, row0, w0, w1, k, t); });
+        }
       } else {
         // NodeEncoder / NodeUpdate.
         // vec layout: [W1^T (n_feat x H) if encoder], (b_l, gamma_l, beta_l) for l = 1..L, b1_edge
@@ -589,18 +665,27 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           GNN_TRACE_W(4);
           l0 = 1;
         }
-        for (int l = l0; l <= L; ++l) {
+        for (int l = l0; l < L; ++l) {
           wait_job();
           GNN_TRACE_W(3 + 2 * l);
-          load_d(v);
           const float* vl = vb + 3 * (l - 1) * H;
-          add_vec(v, vl);
-          ln_relu(v, vl + H, vl + 2 * H);
-          put_a(v);
-          arrive_a(j, seq); next_job();                   // next layer, or the P_s job
+          ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { put_a_chunk(k, t); });
+          tmem_st_wait();
+          arrive_a(j, seq); next_job();                   // next layer
           GNN_TRACE_W(4 + 2 * l);
         }
-        store_t16(p.h, row0, ok && ok0, ok && ok1, v);     // new node state
+        if (l0 <= L) {                                    // last layer: new node state, and A for the P_s job
+          wait_job();
+          GNN_TRACE_W(3 + 2 * L);
+          const float* vl = vb + 3 * (L - 1) * H;
+          const bool w0 = ok && ok0, w1 = ok && ok1;
+          ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) {
+            store_t16_chunk(p.h, row0, w0, w1, k, t);
+            put_a_chunk(k, t);
+          });
+          tmem_st_wait();
+          arrive_a(j, seq); next_job();                   // the P_s job
+        }
         GNN_TRACE_W(11);
         wait_job();                                       // P_s = W_s h (no bias)
         GNN_TRACE_W(12);
