@@ -74,11 +74,16 @@ KERNEL_SOURCES = ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh", "gnn_api.cu")
 
 
 def source_hash() -> str:
+    """First 16 hex digits of a sha256 over the kernel sources' code: `//` comments, trailing
+    blanks and empty lines are left out, so editing a comment does not void a profile."""
     import hashlib
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:
-        with open(os.path.join(ROOT, "paper_2402_09633_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2402_09633_gb300", "csrc", f)) as fh:
+            for line in fh:
+                code = line.split("//", 1)[0].rstrip()
+                if code:
+                    h.update(code.encode() + b"\n")
     return h.hexdigest()[:16]
 
 

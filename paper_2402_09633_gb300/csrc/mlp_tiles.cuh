@@ -11,18 +11,20 @@
 // bf16 splits (v = hi + lo, both bf16) with fp32 accumulation, which keeps the
 // relative product error near 2^-16.
 //
-// Organisation (512 threads = 16 warps, all of them workers):
-//   * two TMEM slots, 8 warps each; slot s works on tile 2p+s of tile pair p,
-//     so while one slot runs its epilogue the tensor core serves the other
-//     (ping-pong);
-//   * there is no dedicated MMA or producer warp: the last of a slot's warps
-//     to publish its part of an A operand issues that slot's MMAs (one thread,
-//     24 tcgen05.mma per layer) and commits them to the slot's mbarrier; when
-//     weights stream through the ring, the second slot to finish with a stage
-//     refills it with a bulk copy;
-//   * a worker warp owns 16 rows of a tile; a quad of threads shares two rows
-//     (each thread a quarter of the columns), reads them from tensor memory
-//     with the 16-lane shapes and does LayerNorm / ReLU in registers.
+// Organisation (640 threads = 20 warps, one CTA per SM; setmaxnreg moves the
+// control warpgroup's registers to the workers):
+//   * two TMEM slots, each a D accumulator and a bf16 hi/lo A operand; slot s
+//     works on tile 2p+s of tile pair p, so while one slot runs its epilogue
+//     the tensor core serves the other (ping-pong);
+//   * control warpgroup (warps 0-3): warp 0 issues the MMAs of whichever slot
+//     has published its next A operand (one thread, 24 tcgen05.mma per layer)
+//     and commits them to the slot's mbarrier; warp 1 loads the weights with
+//     bulk copies (all at once, or streamed through a ring of stages) and
+//     warms L2 with the next tile pair's rows;
+//   * worker warpgroups (warps 4-19), eight warps per slot: a worker warp owns
+//     16 rows of a tile; a quad of threads shares two rows (each thread a
+//     quarter of the columns), reads them from tensor memory with the 16-lane
+//     shapes and does bias / gathers, LayerNorm and ReLU in registers.
 #pragma once
 #include <cstdint>
 #include <cuda_bf16.h>
