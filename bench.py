@@ -224,6 +224,22 @@ def workload_config(w: S.Workload):
             "parallelism": "replicas (one event per GPU per step)"}
 
 
+# ------------------------------------------------------------------ ranks
+def whole_job(local_s: float, local_units: float, world: int, device=None):
+    """Whole-job figures of a step that every rank runs on its own events (replicas, no data-path
+    collective): the slowest rank's time and the units summed over ranks, so throughput is
+    units / time.  All ranks must call it (two all-reduces)."""
+    if world == 1:
+        return local_s, local_units
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([local_s], dtype=torch.float64, device=device)
+    u = torch.tensor([local_units], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
 # ------------------------------------------------------------------ GB300 arm
 def run_gb300(args, rank: int, world: int, local: int):
     import torch
@@ -283,12 +299,9 @@ def run_gb300(args, rank: int, world: int, local: int):
     net.profile(False)
     status = net.status()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    mean_ms = sum(step_ms) / len(step_ms)
-    if world > 1:
-        t = torch.tensor([mean_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        mean_ms = float(t.item())
-    value = world * E / (mean_ms * 1e-3)
+    step_s, job_edges = whole_job(sum(step_ms) / len(step_ms) * 1e-3, E, world, dev)
+    mean_ms = step_s * 1e3
+    value = job_edges / step_s
 
     # end to end through the host-buffer entry point (copies inside the timed region)
     x_h = torch.from_numpy(x_np).pin_memory()
@@ -301,11 +314,7 @@ def run_gb300(args, rank: int, world: int, local: int):
     t0 = time.perf_counter()
     for _ in range(n_e2e):
         net.infer_host(x_h, ei_h, s_h)
-    e2e_s = (time.perf_counter() - t0) / n_e2e
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s, _ = whole_job((time.perf_counter() - t0) / n_e2e, E, world, dev)
     e2e_ok = bool(np.array_equal(s_h.numpy(), scores.cpu().numpy()))
 
     if rank != 0:
@@ -344,13 +353,13 @@ def run_gb300(args, rank: int, world: int, local: int):
             "warmup": args.warmup, "ms_per_step": mean_ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16x3->f32", "data": "synthetic",
             "config": workload_config(w),
-            "events_per_s": value / E * w.n_events,
+            "events_per_s": value / E * w.n_events,                 # every rank scores events of E edges
             "roofline": roofline,
             "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms,
                               "bytes_alg": model["bytes"], "flops_alg": model["flops"]},
             "kernels": groups,
             "cpu_baseline": cpu,
-            "e2e": {"value": world * E / e2e_s, "unit": UNIT,
+            "e2e": {"value": job_edges / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": int(x_np.nbytes + ei_np.nbytes),
                     "d2h_bytes_per_step": int(E * 4), "ms_per_step": e2e_s * 1e3,
                     "matches_device_path": e2e_ok},
