@@ -136,7 +136,8 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
   uint64_t* w_empty = bars + 4 + G::STAGES;          // [STAGES]  both slots' MMAs on a stage completed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * G::STAGES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  volatile int* progress = abort_flag + 1;          // tile pair slot 0's workers are on (L2 prefetch pacing)
+  volatile int* progress = abort_flag + 1;          // [0] tile pair slot 0's workers are on (L2 prefetch pacing)
+                                                    // [1] slot 1 may start (edge kernels: the slots run out of phase)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -150,6 +151,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     for (int s = 0; s < G::STAGES; ++s) { mbar_init(&w_full[s], 1); mbar_init(&w_empty[s], 2); }
     *abort_flag = 0;
     progress[0] = -1;
+    progress[1] = 0;
     fence_mbar_init();
   }
   if (warp == 0) { tmem_alloc(tmem_slot, G::TMEM_COLS); tmem_relinquish(); }
@@ -517,13 +519,27 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
       if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
         // vec layout: [gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]
         if (slot == 0 && ws == 0 && lane == 0) progress[0] = pair;   // paces the L2 prefetcher
+        // The two slots run out of phase: slot 1 starts once slot 0 has released the last MMA of
+        // its first tile, so that one slot's tile change (store, next loads) overlaps the other
+        // slot's MMAs instead of leaving the tensor core idle.  Bounded: it starts anyway after
+        // the wait limit.
+        if (slot == 1 && pair == (int)blockIdx.x) {
+          const uint64_t t0 = global_timer_ns();
+          for (uint32_t it = 0; progress[1] == 0; ++it) {
+            if (*abort_flag || ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs)) break;
+            __nanosleep(64);
+          }
+        }
+        auto release_slot1 = [&]() {
+          if (slot == 0 && pair == (int)blockIdx.x && j == L && ws == 0 && lane == 0) progress[1] = 1;
+        };
         GNN_TRACE_W(0);
         const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
         const int s1 = ok1 ? p.src_sorted[row1] : 0, d1 = ok1 ? p.dst_sorted[row1] : 0;
         load_t16(v, p.e, row0, ok0, ok1);
         GNN_TRACE_W(1);
         put_a(v);
-        arrive_a(j, seq); next_job();                     // job: D = e * W_e^T
+        arrive_a(j, seq); next_job(); release_slot1();                     // job: D = e * W_e^T
         GNN_TRACE_W(2);
         // layer-1 terms of the endpoints, loaded while the MMA runs: P_s[src] + P_d[dst] (P_d carries b1)
 #pragma unroll
@@ -546,7 +562,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         }
         ln_relu(v, vecs, vecs + H);
         put_a(v);
-        arrive_a(j, seq); next_job();
+        arrive_a(j, seq); next_job(); release_slot1();
         GNN_TRACE_W(6);
         for (int l = 2; l <= L; ++l) {
           wait_job();
@@ -555,7 +571,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           const float* vb = vecs + (2 + 3 * (l - 2)) * H;
           add_vec(v, vb);
           ln_relu(v, vb + H, vb + 2 * H);
-          if (l < L) { put_a(v); arrive_a(j, seq); next_job(); }
+          if (l < L) { put_a(v); arrive_a(j, seq); next_job(); release_slot1(); }
           GNN_TRACE_W(6 + 2 * (l - 1));
         }
         if constexpr (KIND == TileKind::EdgeUpdate) {
