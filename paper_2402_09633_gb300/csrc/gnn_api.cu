@@ -14,6 +14,7 @@
 // row pointers) -> node encoder (+ projections) -> edge encoder -> T x (edge
 // update, node update with aggregation + projections) -> classifier.
 #include <cuda_runtime.h>
+#include <algorithm>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -455,7 +456,21 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     push(pl.vecs, head_b, 1);
   }
 
-  for (int i = 0; i < 7; ++i) c->plan[i].vecs.resize(padded_vec_floats((int)c->plan[i].vecs.size()), 0.f);
+  // Every whole H-float segment of a plan's vector block is one per-column vector (bias, gamma,
+  // beta, head weights, a first-layer weight row); the kernels read them in block-pair order:
+  // column 8b + 2q + e at 16*(b/2) + 4q + 2*(b%2) + e.  A trailing partial segment (the head
+  // bias) stays as is.
+  for (int i = 0; i < 7; ++i) {
+    std::vector<float>& v = c->plan[i].vecs;
+    std::vector<float> seg(H);
+    for (size_t base = 0; base + H <= v.size(); base += H) {
+      for (int q = 0; q < 4; ++q)
+        for (int b = 0; b < H / 8; ++b)
+          for (int e = 0; e < 2; ++e) seg[16 * (b / 2) + 4 * q + 2 * (b % 2) + e] = v[base + 8 * b + 2 * q + e];
+      std::copy(seg.begin(), seg.end(), v.begin() + base);
+    }
+    v.resize(padded_vec_floats((int)v.size()), 0.f);
+  }
   err = cudaMalloc(&c->d_mats, packed.size());
   if (err == cudaSuccess) err = cudaMemcpy(c->d_mats, packed.data(), packed.size(), cudaMemcpyHostToDevice);
   for (int i = 0; i < 7 && err == cudaSuccess; ++i) {

@@ -42,10 +42,12 @@ enum class TileKind : int {
 
 constexpr int kThreads = 640;
 // Register split (setmaxnreg): launch at 96 per thread (640 threads x 96 = 61440);
-// the control warpgroup keeps 32, the four worker warpgroups take 112:
-// 128 x 32 + 512 x 112 = 61440.
-constexpr int kControlRegs = 32;
-constexpr int kWorkerRegs = 112;
+// the control warpgroup keeps 64 (the MMA issuer's and the weight producer's
+// loop state must not spill: with ~200 KB of shared memory the L1 is small and
+// a spilled value comes back from L2), the four worker warpgroups take 104:
+// 128 x 64 + 512 x 104 = 61440.
+constexpr int kControlRegs = 64;
+constexpr int kWorkerRegs = 104;
 static_assert(128 * kControlRegs + 512 * kWorkerRegs <= kThreads * 96, "register split exceeds the launch budget");
 constexpr int kTileRows = 128;
 constexpr int kMaxJobs = 8;
@@ -336,6 +338,13 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     auto rm16 = [&](const float* base, int row, int bp) -> const float4* {
       return reinterpret_cast<const float4*>(base + (size_t)row * H + bp * 16 + 2 * cq);
     };
+    // Per-column parameter vectors (bias, gamma, beta, head weights, first-layer weight rows) are
+    // stored by the host in block-pair order: column 8b + 2q + e of an H-vector at index
+    // 16*(b/2) + 4q + 2*(b%2) + e.  The thread with q = lane % 4 reads its two columns of blocks
+    // k and k+1 (k even) as one 16-byte vector, (.x, .y) for block k and (.z, .w) for block k+1,
+    // and the four quad positions read 64 contiguous bytes (no bank conflict).
+    const int qoff = (lane & 3) * 4;
+    auto vq4 = [&](const float* x, int k) { return *reinterpret_cast<const float4*>(x + qoff + 8 * k); };
     // (row r0 quad values of blocks 2bp, 2bp+1) <-> v
     auto put4 = [&](float* v, int bp, int r, const float4& x) {
       v[8 * bp + 2 * r] = x.x; v[8 * bp + 2 * r + 1] = x.y; v[8 * bp + 4 + 2 * r] = x.z; v[8 * bp + 4 + 2 * r + 1] = x.w;
@@ -360,32 +369,19 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
       tmem_st_16x128b_x4(ahi_addr + 16 * k, hi);
       tmem_st_16x128b_x4(alo_addr + 16 * k, lo);
     };
-    // both rows -> bf16 hi/lo A operand (8 blocks per store in the edge kernels, whose
-    // epilogues keep whole rows in registers; 4 in the others, which stream)
+    // both rows -> bf16 hi/lo A operand, four blocks per store pair (keeps the
+    // temporaries at 16 registers next to the row data)
     auto put_a = [&](const float* v) {
-      if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
 #pragma unroll
-        for (int h = 0; h < NB; h += 8) {
-          uint32_t hi[16], lo[16];
-#pragma unroll
-          for (int b = 0; b < 8; ++b) {
-            split_bf16x2(v[4 * (h + b)], v[4 * (h + b) + 1], hi[2 * b], lo[2 * b]);
-            split_bf16x2(v[4 * (h + b) + 2], v[4 * (h + b) + 3], hi[2 * b + 1], lo[2 * b + 1]);
-          }
-          tmem_st_16x128b_x8(ahi_addr + 4 * h, hi);
-          tmem_st_16x128b_x8(alo_addr + 4 * h, lo);
-        }
-      } else {
-#pragma unroll
-        for (int k = 0; k < NB / 4; ++k) put_a_chunk(k, v + 16 * k);
-      }
+      for (int k = 0; k < NB / 4; ++k) put_a_chunk(k, v + 16 * k);
       tmem_st_wait();
     };
     auto add_vec = [&](float* v, const float* b) {
 #pragma unroll
-      for (int k = 0; k < NB; ++k) {
-        const float2 t = *reinterpret_cast<const float2*>(b + 8 * k + cq);
+      for (int k = 0; k < NB; k += 2) {
+        const float4 t = vq4(b, k);
         v[4 * k] += t.x; v[4 * k + 1] += t.y; v[4 * k + 2] += t.x; v[4 * k + 3] += t.y;
+        v[4 * k + 4] += t.z; v[4 * k + 5] += t.w; v[4 * k + 6] += t.z; v[4 * k + 7] += t.w;
       }
     };
     // LayerNorm (biased variance) + ReLU of both rows, in registers.  The host
@@ -403,13 +399,16 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
       const float i0 = rsqrtf(quad_sum(q0) * (1.0f / H) + p.eps);
       const float i1 = rsqrtf(quad_sum(q1) * (1.0f / H) + p.eps);
 #pragma unroll
-      for (int k = 0; k < NB; ++k) {
-        const float2 g = *reinterpret_cast<const float2*>(gamma + 8 * k + cq);
-        const float2 b = *reinterpret_cast<const float2*>(beta + 8 * k + cq);
+      for (int k = 0; k < NB; k += 2) {
+        const float4 g = vq4(gamma, k), b = vq4(beta, k);
         v[4 * k] = fmaxf(fmaf(v[4 * k] * i0, g.x, b.x), 0.f);
         v[4 * k + 1] = fmaxf(fmaf(v[4 * k + 1] * i0, g.y, b.y), 0.f);
         v[4 * k + 2] = fmaxf(fmaf(v[4 * k + 2] * i1, g.x, b.x), 0.f);
         v[4 * k + 3] = fmaxf(fmaf(v[4 * k + 3] * i1, g.y, b.y), 0.f);
+        v[4 * k + 4] = fmaxf(fmaf(v[4 * k + 4] * i0, g.z, b.z), 0.f);
+        v[4 * k + 5] = fmaxf(fmaf(v[4 * k + 5] * i0, g.w, b.w), 0.f);
+        v[4 * k + 6] = fmaxf(fmaf(v[4 * k + 6] * i1, g.z, b.z), 0.f);
+        v[4 * k + 7] = fmaxf(fmaf(v[4 * k + 7] * i1, g.w, b.w), 0.f);
       }
     };
     // LayerNorm + ReLU of D + bias of both rows, streamed from tensor memory in
@@ -425,12 +424,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         for (int c = 0; c < H; c += 64) tmem_ld_16x256b_x8(d_addr + c, t + c / 2);
         tmem_ld_wait();
 #pragma unroll
-        for (int k = 0; k < NB; ++k) {
-          const float2 bb = *reinterpret_cast<const float2*>(bias + 8 * k + cq);
+        for (int k = 0; k < NB; k += 2) {
+          const float4 bb = vq4(bias, k);
           const float a0 = t[4 * k] + bb.x, a1 = t[4 * k + 1] + bb.y;
           const float c0 = t[4 * k + 2] + bb.x, c1 = t[4 * k + 3] + bb.y;
-          q0 = fmaf(a0, a0, fmaf(a1, a1, q0));
-          q1 = fmaf(c0, c0, fmaf(c1, c1, q1));
+          const float a2 = t[4 * k + 4] + bb.z, a3 = t[4 * k + 5] + bb.w;
+          const float c2 = t[4 * k + 6] + bb.z, c3 = t[4 * k + 7] + bb.w;
+          q0 = fmaf(a0, a0, fmaf(a1, a1, fmaf(a2, a2, fmaf(a3, a3, q0))));
+          q1 = fmaf(c0, c0, fmaf(c1, c1, fmaf(c2, c2, fmaf(c3, c3, q1))));
         }
       }
       const float i0 = rsqrtf(quad_sum(q0) * (1.0f / H) + p.eps);
@@ -443,15 +444,17 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         if (k + 1 < NB / 4) tmem_ld_16x256b_x4(d_addr + 32 * (k + 1), t[(k + 1) & 1]);
         float* u = t[k & 1];
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          const int col = 32 * k + 8 * b + cq;
-          const float2 bb = *reinterpret_cast<const float2*>(bias + col);
-          const float2 g = *reinterpret_cast<const float2*>(gamma + col);
-          const float2 be = *reinterpret_cast<const float2*>(beta + col);
+        for (int b = 0; b < 4; b += 2) {
+          const int kb = 4 * k + b;                        // block index
+          const float4 bb = vq4(bias, kb), g = vq4(gamma, kb), be = vq4(beta, kb);
           u[4 * b] = fmaxf(fmaf((u[4 * b] + bb.x) * i0, g.x, be.x), 0.f);
           u[4 * b + 1] = fmaxf(fmaf((u[4 * b + 1] + bb.y) * i0, g.y, be.y), 0.f);
           u[4 * b + 2] = fmaxf(fmaf((u[4 * b + 2] + bb.x) * i1, g.x, be.x), 0.f);
           u[4 * b + 3] = fmaxf(fmaf((u[4 * b + 3] + bb.y) * i1, g.y, be.y), 0.f);
+          u[4 * b + 4] = fmaxf(fmaf((u[4 * b + 4] + bb.z) * i0, g.z, be.z), 0.f);
+          u[4 * b + 5] = fmaxf(fmaf((u[4 * b + 5] + bb.w) * i0, g.w, be.w), 0.f);
+          u[4 * b + 6] = fmaxf(fmaf((u[4 * b + 6] + bb.z) * i1, g.z, be.z), 0.f);
+          u[4 * b + 7] = fmaxf(fmaf((u[4 * b + 7] + bb.w) * i1, g.w, be.w), 0.f);
         }
         emit(k, u);
         if (k + 1 < NB / 4) tmem_ld_wait();
@@ -489,9 +492,10 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         tmem_ld_wait();
         if (bias) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const float2 bb = *reinterpret_cast<const float2*>(bias + c + 8 * k + cq);
+          for (int k = 0; k < 4; k += 2) {
+            const float4 bb = vq4(bias, c / 8 + k);
             t[4 * k] += bb.x; t[4 * k + 1] += bb.y; t[4 * k + 2] += bb.x; t[4 * k + 3] += bb.y;
+            t[4 * k + 4] += bb.z; t[4 * k + 5] += bb.w; t[4 * k + 6] += bb.z; t[4 * k + 7] += bb.w;
           }
         }
 #pragma unroll
@@ -541,24 +545,38 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         put_a(v);
         arrive_a(j, seq); next_job(); release_slot1();                     // job: D = e * W_e^T
         GNN_TRACE_W(2);
-        // layer-1 terms of the endpoints, loaded while the MMA runs: P_s[src] + P_d[dst] (P_d carries b1)
+        // layer-1 terms of the endpoints, loaded while the MMA runs: P_s[src] + P_d[dst] (P_d carries
+        // b1).  P_s rows go straight into v; P_d rows follow two block pairs at a time, so at most
+        // 16 registers of loads are in flight next to the row data.
 #pragma unroll
         for (int bp = 0; bp < NB / 2; ++bp) {
-          const float4 a0 = *rm16(p.ps, s0, bp), b0 = *rm16(p.pd, d0, bp);
-          const float4 a1 = *rm16(p.ps, s1, bp), b1 = *rm16(p.pd, d1, bp);
-          put4(v, bp, 0, make_float4(a0.x + b0.x, a0.y + b0.y, a0.z + b0.z, a0.w + b0.w));
-          put4(v, bp, 1, make_float4(a1.x + b1.x, a1.y + b1.y, a1.z + b1.z, a1.w + b1.w));
+          put4(v, bp, 0, *rm16(p.ps, s0, bp));
+          put4(v, bp, 1, *rm16(p.ps, s1, bp));
+        }
+#pragma unroll
+        for (int g = 0; g < NB / 2; g += 2) {
+          float4 b[4];
+#pragma unroll
+          for (int k = 0; k < 2; ++k) { b[2 * k] = *rm16(p.pd, d0, g + k); b[2 * k + 1] = *rm16(p.pd, d1, g + k); }
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            const float4 x0 = get4(v, g + k, 0), x1 = get4(v, g + k, 1);
+            const float4& y0 = b[2 * k];
+            const float4& y1 = b[2 * k + 1];
+            put4(v, g + k, 0, make_float4(x0.x + y0.x, x0.y + y0.y, x0.z + y0.z, x0.w + y0.w));
+            put4(v, g + k, 1, make_float4(x1.x + y1.x, x1.y + y1.y, x1.z + y1.z, x1.w + y1.w));
+          }
         }
         GNN_TRACE_W(3);
         wait_job();
         GNN_TRACE_W(5);
 #pragma unroll
-        for (int c = 0; c < H; c += 64) {                 // v += D
-          float t[32];
-          tmem_ld_16x256b_x8(d_addr + c, t);
+        for (int c = 0; c < H; c += 32) {                 // v += D, 32 columns per TMEM round trip
+          float t[16];
+          tmem_ld_16x256b_x4(d_addr + c, t);
           tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[c / 2 + i] += t[i];
+          for (int i = 0; i < 16; ++i) v[c / 2 + i] += t[i];
         }
         ln_relu(v, vecs, vecs + H);
         put_a(v);
@@ -581,10 +599,10 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           const float* wo = vecs + (2 + 3 * (L - 1)) * H;
           float z0 = 0.f, z1 = 0.f;
 #pragma unroll
-          for (int k = 0; k < NB; ++k) {
-            const float2 w = *reinterpret_cast<const float2*>(wo + 8 * k + cq);
-            z0 = fmaf(v[4 * k], w.x, fmaf(v[4 * k + 1], w.y, z0));
-            z1 = fmaf(v[4 * k + 2], w.x, fmaf(v[4 * k + 3], w.y, z1));
+          for (int k = 0; k < NB; k += 2) {
+            const float4 w = vq4(wo, k);
+            z0 = fmaf(v[4 * k], w.x, fmaf(v[4 * k + 1], w.y, fmaf(v[4 * k + 4], w.z, fmaf(v[4 * k + 5], w.w, z0))));
+            z1 = fmaf(v[4 * k + 2], w.x, fmaf(v[4 * k + 3], w.y, fmaf(v[4 * k + 6], w.z, fmaf(v[4 * k + 7], w.w, z1))));
           }
           z0 = quad_sum(z0) + wo[H];
           z1 = quad_sum(z1) + wo[H];
@@ -613,13 +631,16 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         }
         const float* vb = vecs + 2 * H;
 #pragma unroll
-        for (int k = 0; k < NB; ++k) {
-          const float2 w0 = *reinterpret_cast<const float2*>(vecs + 8 * k + cq);
-          const float2 w1 = *reinterpret_cast<const float2*>(vecs + H + 8 * k + cq);
+        for (int k = 0; k < NB; k += 2) {
+          const float4 w0 = vq4(vecs, k), w1 = vq4(vecs + H, k);
           v[4 * k] = fmaf(w1.x, f[0][1], w0.x * f[0][0]);
           v[4 * k + 1] = fmaf(w1.y, f[0][1], w0.y * f[0][0]);
           v[4 * k + 2] = fmaf(w1.x, f[1][1], w0.x * f[1][0]);
           v[4 * k + 3] = fmaf(w1.y, f[1][1], w0.y * f[1][0]);
+          v[4 * k + 4] = fmaf(w1.z, f[0][1], w0.z * f[0][0]);
+          v[4 * k + 5] = fmaf(w1.w, f[0][1], w0.w * f[0][0]);
+          v[4 * k + 6] = fmaf(w1.z, f[1][1], w0.z * f[1][0]);
+          v[4 * k + 7] = fmaf(w1.w, f[1][1], w0.w * f[1][0]);
         }
         add_vec(v, vb);
         ln_relu(v, vb + H, vb + 2 * H);
@@ -650,10 +671,12 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
             const float x0 = ok0 ? p.x[(size_t)row0 * p.x_stride + k] : 0.f;
             const float x1 = ok1 ? p.x[(size_t)row1 * p.x_stride + k] : 0.f;
 #pragma unroll
-            for (int b = 0; b < NB; ++b) {
-              const float2 w = *reinterpret_cast<const float2*>(vecs + k * H + 8 * b + cq);
+            for (int b = 0; b < NB; b += 2) {
+              const float4 w = vq4(vecs + k * H, b);
               v[4 * b] = fmaf(w.x, x0, v[4 * b]); v[4 * b + 1] = fmaf(w.y, x0, v[4 * b + 1]);
               v[4 * b + 2] = fmaf(w.x, x1, v[4 * b + 2]); v[4 * b + 3] = fmaf(w.y, x1, v[4 * b + 3]);
+              v[4 * b + 4] = fmaf(w.z, x0, v[4 * b + 4]); v[4 * b + 5] = fmaf(w.w, x0, v[4 * b + 5]);
+              v[4 * b + 6] = fmaf(w.z, x1, v[4 * b + 6]); v[4 * b + 7] = fmaf(w.w, x1, v[4 * b + 7]);
             }
           }
           add_vec(v, vb);
@@ -667,17 +690,13 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           put_a(v);
           arrive_a(j, seq); next_job();                   // job: D = h * W_h^T
           GNN_TRACE_W(1);
-          if (ws == 0 && lane == 0) {
-            const int nt = tile + 2 * (int)gridDim.x;
-            if (nt < p.n_tiles) {
-              prefetch_l2_bulk(p.h + (size_t)nt * kTileRows * H, kTileRows * H * 4);
-              prefetch_l2_bulk(p.agg + (size_t)nt * kTileRows * H, kTileRows * H * 4);
-            }
-          }
-          load_t16(v, p.agg, row0, ok0, ok1);              // a_j, summed by the aggregation kernel
+          // The aggregate rows are loaded only after the first job completed: a burst of global
+          // loads from a slot's warps while its MMAs run slows those MMAs several-fold (the loads
+          // compete with the tensor core's operand reads in the SM's memory pipeline).
           GNN_TRACE_W(2);
           wait_job();                                     // A free again
           GNN_TRACE_W(3);
+          load_t16(v, p.agg, row0, ok0, ok1);              // a_j, summed by the aggregation kernel
           put_a(v);
           arrive_a(j, seq); next_job();                   // job: D += a * W_a^T
           GNN_TRACE_W(4);
