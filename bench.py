@@ -49,7 +49,9 @@ def step_model(w: S.Workload):
     """Algorithmic bytes and flops of one step (whole path) and of the two iteration kernels."""
     m, ev = w.model, w.event
     N, E = ev.n_nodes * w.n_events, ev.n_edges * w.n_events
-    H, T, L, Fn, s = m.hidden, m.n_iters, m.mlp_layers, m.n_node_feat, 4
+    bf16 = m.precision == S.PRECISION_BF16
+    # s: bytes of a stored activation (the step model); the projections P_s, P_d are fp32 in both models
+    H, T, L, Fn, s, sp = m.hidden, m.n_iters, m.mlp_layers, m.n_node_feat, (2 if bf16 else 4), 4
     bytes_step = (32 * E + 4 * N + 4 * Fn * N + (E + N) * H * s
                   + T * ((3 * E + 2 * N) * H * s + 4 * E + 4 * N) + (2 * E + N) * H * s + 8 * E)
     mac_edge_iter = E * H * H * L                           # e * W_e, then L-1 H x H layers
@@ -58,12 +60,11 @@ def step_model(w: S.Workload):
                       + N * (Fn * H + H * H * (L - 1) + 2 * H * H)      # node encoder + projections
                       + E * (2 * H + H * H * (L - 1))                   # edge encoder
                       + E * (H * H * L + H))                            # classifier (+ head)
-    edge_update = {"bytes": E * (3 * H * s + 8) + N * H * s, "flops": 2 * mac_edge_iter,
-                   "bytes_note": "per edge: e read + e write + gathered W_s h_src row + 2 indices; "
-                                 "per node: W_d h_dst + b1 row"}
-    node_update = {"bytes": E * H * s + N * (5 * H * s + 8), "flops": 2 * mac_node_iter,
-                   "bytes_note": "per edge: message row of the CSR segment sum; per node: h read+write, "
-                                 "P_s/P_d write, its first-layer row, row pointers"}
+    edge_update = {"bytes": E * (2 * H * s + H * sp + 8) + N * H * sp, "flops": 2 * mac_edge_iter,
+                   "bytes_note": "per edge: e read + e write + gathered W_s h_src row (fp32) + 2 indices; "
+                                 "per node: W_d h_dst + b1 row (fp32)"}
+    node_update = {"bytes": N * (3 * H * s + 2 * H * sp), "flops": 2 * mac_node_iter,
+                   "bytes_note": "per node: h and a read, h write, P_s and P_d (fp32) write"}
     return {"bytes": bytes_step, "flops": flops_step, "N": N, "E": E,
             "edge_update": edge_update, "node_update": node_update}
 
@@ -171,11 +172,12 @@ def oracle_sample(w: S.Workload, scale: float, seed: int = 0):
 def time_oracle(w: S.Workload, scale: float, repeats: int = 1):
     from oracle import gnn_oracle as O       # CPU baseline leg only
     W, x, ei = oracle_sample(w, scale)
-    O.forward(W, x[:50], ei[:, :0], w.model.n_iters)          # import / allocator warm-up
+    bf16 = w.model.precision == S.PRECISION_BF16
+    O.forward(W, x[:50], ei[:, :0], w.model.n_iters, bf16=bf16)          # import / allocator warm-up
     times = []
     for _ in range(repeats):
         t0 = time.perf_counter()
-        O.forward(W, x, ei, w.model.n_iters, w.model.ln_eps)
+        O.forward(W, x, ei, w.model.n_iters, w.model.ln_eps, bf16=bf16)
         times.append(time.perf_counter() - t0)
     return ei.shape[1], x.shape[0], times
 
@@ -336,7 +338,8 @@ def run_gb300(args, rank: int, world: int, local: int):
                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": profiled_traffic(dom),
                     "peak_source": f"{peak_src} (hbm_gbs, copy burst) -- of {peak_src}",
                     "bytes_per_launch": dom_model["bytes"], "avg_launch_ms": dom_avg_s * 1e3,
-                    "tensor_tflops_executed": 3 * dom_model["flops"] / dom_avg_s / 1e12}
+                    "tensor_tflops_executed": (1 if w.model.precision == S.PRECISION_BF16 else 3)
+                                              * dom_model["flops"] / dom_avg_s / 1e12}
     t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9),
                           model["flops"] / (peaks["bf16_tflops"] * 1e12))
     total_launches = sum(v["launches"] for v in kernels_only.values())
@@ -351,7 +354,8 @@ def run_gb300(args, rank: int, world: int, local: int):
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": mean_ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16x3->f32", "data": "synthetic",
+            "vs_baseline": None, "dtype": "bf16->f32" if w.model.precision == S.PRECISION_BF16 else "bf16x3->f32",
+            "data": "synthetic",
             "config": workload_config(w),
             "events_per_s": value / E * w.n_events,                 # every rank scores events of E edges
             "roofline": roofline,

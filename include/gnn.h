@@ -52,7 +52,8 @@ enum gnn_status_code {
 
 enum gnn_precision {
   GNN_PRECISION_FP32 = 0,      /* fp32 weights and state; products as three bf16 pieces */
-  GNN_PRECISION_BF16 = 1,      /* reserved: bf16 weights and state (not built yet) */
+  GNN_PRECISION_BF16 = 1,      /* bf16 weights, activations and stored states (h, e, a); fp32
+                                  accumulation and LayerNorm; the blob's values must be bf16 */
 };
 
 /* Model configuration (must equal the blob header). */
@@ -164,7 +165,7 @@ const char* gnn_error_string(int code);
  * into caller device memory `dst` of at least `bytes` bytes (enqueued on
  * `stream`).  which: 0 rowptr int32 [N+1], 1 perm int32 [E] (CSR slot ->
  * input edge id), 2 src_sorted int32 [E], 3 node state h, 4 edge state e (CSR
- * order).  The states are float32 in the row-tiled layout of the kernels:
+ * order).  The states are float32 (bfloat16 for GNN_PRECISION_BF16) in the row-tiled layout of the kernels:
  * R = rows rounded up to a multiple of 128, element (r, c) at index
  * ((r / 128) * (H / 16) + bp) * 2048 + (r % 128) * 16 + x, R * H floats, where
  * b = c / 8, bp = b / 2 and x = 4 * ((c % 8) / 2) + 2 * (b % 2) + c % 2.

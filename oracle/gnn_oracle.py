@@ -27,6 +27,16 @@ features is rounded to float32 and the wrap into (-1, 1] (units of pi; exact
 +-1 maps to +1) is decided on that float32 value, so the oracle and a float32
 kernel take the same wrap decision.
 
+The bf16 model (bf16 weights and activations, wider accumulation) is the same
+network with every activation rounded to the nearest bfloat16 (ties to even):
+the output of every MLP layer (so every input of a Linear layer after the
+first, and the stored states h and e) and the aggregate a_j.  Its weights are
+bf16 values by construction (the caller passes them); the raw inputs x and the
+edge features stay float32.  `forward(..., bf16=True)` evaluates it; the
+`dtype` argument chooses the accumulation precision (float64 by default;
+float32 gives a second, equally valid evaluation of the bf16 model, used to
+measure how far rounding-order differences alone move its logits).
+
 Every routine works on plain numpy arrays; the matrix product, argsort and
 np.add.at are the only library primitives used.
 """
@@ -48,13 +58,28 @@ def relu(v: np.ndarray) -> np.ndarray:
     return np.maximum(v, 0.0)
 
 
-def mlp(v: np.ndarray, layers, eps: float) -> np.ndarray:
-    """Stack of Linear -> LayerNorm -> ReLU layers; `layers` = [(W [out,in], b, gamma, beta)]."""
-    v = np.asarray(v, dtype=np.float64)
+def round_bf16(a: np.ndarray) -> np.ndarray:
+    """Nearest bfloat16 value (8 significant bits, ties to even) of each element, as float64.
+
+    Written from the format's definition: a = m * 2^e with 0.5 <= |m| < 1; the
+    nearest value with 8 significant bits is rint(m * 2^8) * 2^(e - 8), where
+    rint rounds halfway cases to even.  (Magnitudes here stay far from the
+    bfloat16 overflow and subnormal ranges.)"""
+    a = np.asarray(a, dtype=np.float64)
+    m, e = np.frexp(a)
+    return np.ldexp(np.rint(m * 256.0), e - 8)
+
+
+def mlp(v: np.ndarray, layers, eps: float, act=None, dtype=np.float64) -> np.ndarray:
+    """Stack of Linear -> LayerNorm -> ReLU layers; `layers` = [(W [out,in], b, gamma, beta)].
+    `act`, when given, is applied to every layer's output (the bf16 model rounds there)."""
+    v = np.asarray(v, dtype=dtype)
     for (W, b, g, be) in layers:
-        W = np.asarray(W, np.float64)
-        v = relu(layer_norm(v @ W.T + np.asarray(b, np.float64),
-                            np.asarray(g, np.float64), np.asarray(be, np.float64), eps))
+        W = np.asarray(W, dtype)
+        v = relu(layer_norm(v @ W.T + np.asarray(b, dtype),
+                            np.asarray(g, dtype), np.asarray(be, dtype), dtype(eps)))
+        if act is not None:
+            v = act(v).astype(dtype)
     return v
 
 
@@ -86,9 +111,9 @@ def csr_by_destination(src: np.ndarray, dst: np.ndarray, n_nodes: int):
     return rowptr, np.asarray(src, np.int64)[perm], perm
 
 
-def aggregate(m: np.ndarray, dst: np.ndarray, n_nodes: int) -> np.ndarray:
+def aggregate(m: np.ndarray, dst: np.ndarray, n_nodes: int, dtype=np.float64) -> np.ndarray:
     """a_j = sum of the messages of all edges whose destination is j (0 if none)."""
-    a = np.zeros((n_nodes, m.shape[1]), dtype=np.float64)
+    a = np.zeros((n_nodes, m.shape[1]), dtype=dtype)
     np.add.at(a, np.asarray(dst, np.int64), m)
     return a
 
@@ -100,26 +125,31 @@ def sigmoid(z: np.ndarray) -> np.ndarray:
 
 
 def forward(weights: dict, x: np.ndarray, edge_index: np.ndarray, n_iters: int,
-            eps: float = 1e-5, return_logits: bool = False, return_states: bool = False):
+            eps: float = 1e-5, return_logits: bool = False, return_states: bool = False,
+            bf16: bool = False, dtype=np.float64):
     """Edge scores (input edge order) of the interaction network on one hit graph.
 
     `weights` maps each MLP name to its [(W, b, gamma, beta)] layers, plus
     'head_w' [H] and 'head_b' [1].  `edge_index` is [2, E] (row 0 source, row 1
-    destination).  Returns scores (and logits / final states on request)."""
+    destination).  `bf16` evaluates the bf16 model (activations rounded to
+    bfloat16, see the module doc); `dtype` is the accumulation precision.
+    Returns scores (and logits / final states on request)."""
     x = np.asarray(x, dtype=np.float32)
     src = np.asarray(edge_index[0], dtype=np.int64)
     dst = np.asarray(edge_index[1], dtype=np.int64)
     n_nodes = x.shape[0]
-    f = edge_features(x, src, dst).astype(np.float64)
-    h = mlp(x.astype(np.float64), weights["node_encoder"], eps)
-    e = mlp(f, weights["edge_encoder"], eps)
+    act = round_bf16 if bf16 else None
+    keep = (lambda v: round_bf16(v).astype(dtype)) if bf16 else (lambda v: v)
+    f = edge_features(x, src, dst).astype(dtype)
+    h = mlp(x.astype(dtype), weights["node_encoder"], eps, act, dtype)
+    e = mlp(f, weights["edge_encoder"], eps, act, dtype)
     for _ in range(n_iters):
-        m = mlp(np.concatenate([h[src], h[dst], e], axis=1), weights["edge_network"], eps)
+        m = mlp(np.concatenate([h[src], h[dst], e], axis=1), weights["edge_network"], eps, act, dtype)
         e = m
-        a = aggregate(m, dst, n_nodes)
-        h = mlp(np.concatenate([h, a], axis=1), weights["node_network"], eps)
-    c = mlp(np.concatenate([h[src], h[dst], e], axis=1), weights["edge_classifier"], eps)
-    logits = c @ np.asarray(weights["head_w"], np.float64) + float(np.asarray(weights["head_b"])[0])
+        a = keep(aggregate(m, dst, n_nodes, dtype))
+        h = mlp(np.concatenate([h, a], axis=1), weights["node_network"], eps, act, dtype)
+    c = mlp(np.concatenate([h[src], h[dst], e], axis=1), weights["edge_classifier"], eps, act, dtype)
+    logits = (c @ np.asarray(weights["head_w"], dtype) + dtype(np.asarray(weights["head_b"])[0])).astype(np.float64)
     scores = sigmoid(logits)
     out = [scores]
     if return_logits:

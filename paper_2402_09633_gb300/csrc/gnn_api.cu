@@ -63,7 +63,8 @@ struct gnn_ctx {
   int *keys_a = nullptr, *keys_b = nullptr, *vals_a = nullptr, *vals_b = nullptr, *src_c = nullptr;
   int *hist = nullptr, *perm = nullptr, *src_sorted = nullptr, *dst_sorted = nullptr, *rowptr = nullptr;
   int* key_sorted = nullptr;
-  float *e = nullptr, *h = nullptr, *ps = nullptr, *pd = nullptr, *agg = nullptr;
+  void *e = nullptr, *h = nullptr, *agg = nullptr;  // stored states (fp32 or bf16 per precision)
+  float *ps = nullptr, *pd = nullptr;
   int64_t last_nodes = 0, last_edges = 0;
   // staging for gnn_infer_host
   void* stage = nullptr;
@@ -104,17 +105,20 @@ inline size_t swizzled_offset(int H, int n, int k) {
          (((kk / 8) ^ (n % 8)) * 16) + (kk % 8) * 2;
 }
 
-// Pack columns [col0, col0+H) of W [H, ld] into hi/lo bf16 parts.
-void pack_block(const float* W, int ld, int col0, int H, uint8_t* out) {
+// Pack columns [col0, col0+H) of W [H, ld] into hi/lo bf16 parts (fp32 model), or
+// into the single bf16 part (bf16 model: W holds bf16 values, hi == W exactly).
+void pack_block(const float* W, int ld, int col0, int H, bool with_lo, uint8_t* out) {
   const size_t part = (size_t)H * H * 2;
   for (int n = 0; n < H; ++n)
     for (int k = 0; k < H; ++k) {
       const float v = W[(size_t)n * ld + col0 + k];
       const uint16_t hi = f32_to_bf16_rne(v);
-      const uint16_t lo = f32_to_bf16_rne(v - bf16_to_f32(hi));
       const size_t off = swizzled_offset(H, n, k);
       std::memcpy(out + off, &hi, 2);
-      std::memcpy(out + part + off, &lo, 2);
+      if (with_lo) {
+        const uint16_t lo = f32_to_bf16_rne(v - bf16_to_f32(hi));
+        std::memcpy(out + part + off, &lo, 2);
+      }
     }
 }
 
@@ -145,23 +149,23 @@ void prof_end(gnn_ctx* c, int idx, cudaStream_t st) {
   if (idx >= 0) cudaEventRecord(c->prof[idx].b, st);
 }
 
-template <TileKind K, int H>
+template <TileKind K, int H, bool BF>
 cudaError_t set_smem_attr() {
-  return cudaFuncSetAttribute(mlp_tile_kernel<K, H>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(mlp_tile_kernel<K, H, BF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               227 * 1024);
 }
 
-template <int H>
+template <int H, bool BF>
 cudaError_t set_all_attrs() {
   cudaError_t e;
-  if ((e = set_smem_attr<TileKind::NodeEncoder, H>()) != cudaSuccess) return e;
-  if ((e = set_smem_attr<TileKind::EdgeEncoder, H>()) != cudaSuccess) return e;
-  if ((e = set_smem_attr<TileKind::EdgeUpdate, H>()) != cudaSuccess) return e;
-  if ((e = set_smem_attr<TileKind::NodeUpdate, H>()) != cudaSuccess) return e;
-  return set_smem_attr<TileKind::Classifier, H>();
+  if ((e = set_smem_attr<TileKind::NodeEncoder, H, BF>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::EdgeEncoder, H, BF>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::EdgeUpdate, H, BF>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::NodeUpdate, H, BF>()) != cudaSuccess) return e;
+  return set_smem_attr<TileKind::Classifier, H, BF>();
 }
 
-template <TileKind K, int H>
+template <TileKind K, int H, bool BF>
 void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st) {
   p.n_jobs = pl.n_jobs;
   for (int j = 0; j < kMaxJobs; ++j) { p.job_mat[j] = pl.job_mat[j]; p.job_acc[j] = pl.job_acc[j]; }
@@ -171,7 +175,7 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
   p.mat_bytes = c->mat_bytes;
   p.n_tiles = (p.n_rows + kTileRows - 1) / kTileRows;
   if (p.n_tiles == 0) return;
-  uint32_t smem = tile_smem_bytes<H>(p.n_vec_floats);
+  uint32_t smem = tile_smem_bytes<H, BF>(p.n_vec_floats);
   if (smem < 120 * 1024) smem = 120 * 1024;           // one CTA per SM (it owns the TMEM)
   const int pairs = (p.n_tiles + 1) / 2;
   const int grid = pairs < c->n_sm ? pairs : c->n_sm;
@@ -180,11 +184,11 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
 #endif
   static const int group[5] = {1, 2, 3, 4, 5};      // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier
   const int pr = prof_begin(c, group[(int)K], 1, st);
-  mlp_tile_kernel<K, H><<<grid, kThreads, smem, st>>>(p);
+  mlp_tile_kernel<K, H, BF><<<grid, kThreads, smem, st>>>(p);
   prof_end(c, pr, st);
 }
 
-template <int H>
+template <int H, bool BF>
 int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStream_t st) {
   TileParams p{};
   p.n_nodes = N;
@@ -203,23 +207,25 @@ int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStr
   const int T = c->cfg.n_iters;
 
   TileParams pn = p; pn.n_rows = N; pn.n_feat = c->cfg.n_node_feat;
-  launch_tile<TileKind::NodeEncoder, H>(c, c->plan[T > 0 ? 0 : 1], pn, st);
+  launch_tile<TileKind::NodeEncoder, H, BF>(c, c->plan[T > 0 ? 0 : 1], pn, st);
   TileParams pe = p; pe.n_rows = E; pe.n_feat = 2;
-  launch_tile<TileKind::EdgeEncoder, H>(c, c->plan[2], pe, st);
+  launch_tile<TileKind::EdgeEncoder, H, BF>(c, c->plan[2], pe, st);
   for (int t = 1; t <= T; ++t) {
-    launch_tile<TileKind::EdgeUpdate, H>(c, c->plan[3], pe, st);
+    launch_tile<TileKind::EdgeUpdate, H, BF>(c, c->plan[3], pe, st);
     {
       const int pr = prof_begin(c, 7, 1, st);
       constexpr int npb = agg_nodes_per_block<H>();
-      aggregate_kernel<H><<<(N + npb - 1) / npb, 256, 0, st>>>(c->e, c->rowptr, N, c->agg);
+      aggregate_kernel<H, BF><<<(N + npb - 1) / npb, 256, 0, st>>>(c->e, c->rowptr, N, c->agg);
       prof_end(c, pr, st);
     }
-    launch_tile<TileKind::NodeUpdate, H>(c, c->plan[t < T ? 4 : 5], pn, st);
+    launch_tile<TileKind::NodeUpdate, H, BF>(c, c->plan[t < T ? 4 : 5], pn, st);
   }
-  launch_tile<TileKind::Classifier, H>(c, c->plan[6], pe, st);
+  launch_tile<TileKind::Classifier, H, BF>(c, c->plan[6], pe, st);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
+
+int64_t state_bytes(const gnn_ctx* c) { return c->cfg.precision == GNN_PRECISION_BF16 ? 2 : 4; }
 
 void free_workspace(gnn_ctx* c) {
   if (c->ws) cudaFree(c->ws);
@@ -238,8 +244,9 @@ int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
   // edge and node state use the row-tiled layout: rows padded to whole 128-row tiles
   const int64_t e_pad = (e + kTileRows - 1) / kTileRows * kTileRows;
   const int64_t n_pad = (n + kTileRows - 1) / kTileRows * kTileRows;
+  const int64_t se = state_bytes(c);                   // stored-state element: fp32 or bf16
   const int64_t total = 8 * sz_e_int + al(4 * 256 * (rs_tiles > 0 ? rs_tiles : 1)) + al(4 * (n + 1)) +
-                        al(4 * e_pad * H) + 2 * al(4 * n_pad * H) + 2 * al(4 * n * H);
+                        al(se * e_pad * H) + 2 * al(se * n_pad * H) + 2 * al(4 * n * H);
   free_workspace(c);
   void* ws = nullptr;
   cudaError_t err = cudaMalloc(&ws, (size_t)total);
@@ -253,9 +260,9 @@ int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
   c->src_sorted = (int*)take(4 * e); c->dst_sorted = (int*)take(4 * e);
   c->hist = (int*)take(4 * 256 * (rs_tiles > 0 ? rs_tiles : 1));
   c->rowptr = (int*)take(4 * (n + 1));
-  c->e = (float*)take(4 * e_pad * H);
-  c->h = (float*)take(4 * n_pad * H);
-  c->agg = (float*)take(4 * n_pad * H);
+  c->e = take(se * e_pad * H);
+  c->h = take(se * n_pad * H);
+  c->agg = take(se * n_pad * H);
   c->ps = (float*)take(4 * n * H);
   c->pd = (float*)take(4 * n * H);
   c->cap_nodes = n;
@@ -316,7 +323,7 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
   const int H = cfg->hidden, L = cfg->mlp_layers, Fn = cfg->n_node_feat;
   if (cfg->version != 1 || (H != 64 && H != 128) || L < 2 || L > 4 || Fn < 2 || Fn > 16 ||
       cfg->n_edge_feat != 2 || cfg->n_iters < 0 || cfg->n_iters > 64 ||
-      cfg->precision != GNN_PRECISION_FP32 || !(cfg->ln_eps > 0.f))
+      (cfg->precision != GNN_PRECISION_FP32 && cfg->precision != GNN_PRECISION_BF16) || !(cfg->ln_eps > 0.f))
     return GNN_ERR_INVALID_ARG;
   if (weights_bytes < (size_t)kHeaderBytes) return GNN_ERR_BAD_WEIGHTS;
   const uint8_t* blob = (const uint8_t*)weights_host;
@@ -352,9 +359,12 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
   // rows (W' = (I - 11^T/H) W, b' = b - mean(b)).  The kernels then receive
   // zero-mean pre-activations and compute only the variance.  Centred copies
   // are kept in `centred` and the Layer pointers redirected to them.
+  // The bf16 model keeps its weights as given (bf16 values): centring would take them off the
+  // bf16 grid, so its kernels subtract the LayerNorm mean themselves.
+  const bool bf = cfg->precision == GNN_PRECISION_BF16;
   std::vector<std::vector<float>> centred;
   centred.reserve(2 * N_MLP * L);
-  for (int m = 0; m < N_MLP; ++m)
+  for (int m = 0; m < N_MLP && !bf; ++m)
     for (int l = 0; l < L; ++l) {
       Layer& ly = lay[m][l];
       std::vector<float> Wc((size_t)H * ly.in), bc(H);
@@ -379,7 +389,9 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
   c->cfg = *cfg;
   cudaError_t err = cudaGetDevice(&c->device);
   if (err == cudaSuccess) err = cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
-  if (err == cudaSuccess) err = (H == 128) ? set_all_attrs<128>() : set_all_attrs<64>();
+  if (err == cudaSuccess)
+    err = bf ? ((H == 128) ? set_all_attrs<128, true>() : set_all_attrs<64, true>())
+             : ((H == 128) ? set_all_attrs<128, false>() : set_all_attrs<64, false>());
   if (err != cudaSuccess) { delete c; return cuda_fail(err); }
 
   // matrices
@@ -393,10 +405,10 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
   int deep[N_MLP][4];
   for (int m = 0; m < N_MLP; ++m)
     for (int l = 1; l < L; ++l) deep[m][l] = add_mat(&lay[m][l], 0);
-  c->mat_bytes = 2u * H * H * 2u;
+  c->mat_bytes = (bf ? 1u : 2u) * H * H * 2u;
   std::vector<uint8_t> packed((size_t)c->mat_bytes * mats.size());
   for (size_t i = 0; i < mats.size(); ++i)
-    pack_block(mats[i].first->W, mats[i].first->in, mats[i].second, H, packed.data() + i * c->mat_bytes);
+    pack_block(mats[i].first->W, mats[i].first->in, mats[i].second, H, !bf, packed.data() + i * c->mat_bytes);
 
   // kernel plans
   auto jobs = [](KernelPlan& pl, std::initializer_list<int> ids, int acc_mask = 0) {
@@ -510,8 +522,12 @@ int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, 
   if (rc != GNN_OK) return rc;
   ctx->last_nodes = N;
   ctx->last_edges = E;
-  return ctx->cfg.hidden == 128 ? run_network<128>(ctx, node_feats, N, E, edge_scores, st)
-                                : run_network<64>(ctx, node_feats, N, E, edge_scores, st);
+  const bool bf = ctx->cfg.precision == GNN_PRECISION_BF16;
+  if (ctx->cfg.hidden == 128)
+    return bf ? run_network<128, true>(ctx, node_feats, N, E, edge_scores, st)
+              : run_network<128, false>(ctx, node_feats, N, E, edge_scores, st);
+  return bf ? run_network<64, true>(ctx, node_feats, N, E, edge_scores, st)
+            : run_network<64, false>(ctx, node_feats, N, E, edge_scores, st);
 }
 
 int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
@@ -617,8 +633,8 @@ int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_
     case 0: src = ctx->rowptr; need = 4 * (size_t)(N + 1); break;
     case 1: src = ctx->perm; need = 4 * (size_t)E; break;
     case 2: src = ctx->src_sorted; need = 4 * (size_t)E; break;
-    case 3: src = ctx->h; need = 4 * (size_t)((N + kTileRows - 1) / kTileRows * kTileRows * H); break;
-    case 4: src = ctx->e; need = 4 * (size_t)((E + kTileRows - 1) / kTileRows * kTileRows * H); break;
+    case 3: src = ctx->h; need = state_bytes(ctx) * (size_t)((N + kTileRows - 1) / kTileRows * kTileRows * H); break;
+    case 4: src = ctx->e; need = state_bytes(ctx) * (size_t)((E + kTileRows - 1) / kTileRows * kTileRows * H); break;
     default: return GNN_ERR_INVALID_ARG;
   }
   if (bytes < need) return GNN_ERR_INVALID_ARG;

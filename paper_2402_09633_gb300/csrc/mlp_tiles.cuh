@@ -7,9 +7,14 @@
 // followed by an epilogue in registers (bias or gathered projections,
 // LayerNorm, ReLU) that writes the next layer's A back into tensor memory.
 //
-// Precision: fp32 model, every product evaluated as hi*hi + hi*lo + lo*hi of
-// bf16 splits (v = hi + lo, both bf16) with fp32 accumulation, which keeps the
-// relative product error near 2^-16.
+// Precision (template parameter BF):
+//   * fp32 model (BF = false): fp32 weights and states; every product is
+//     evaluated as hi*hi + hi*lo + lo*hi of bf16 splits (v = hi + lo, both bf16)
+//     with fp32 accumulation, which keeps the relative product error near 2^-16;
+//   * bf16 model (BF = true): bf16 weights, bf16 activations and stored states
+//     (e, h, a), one bf16 product per K step, fp32 accumulation and fp32
+//     LayerNorm; the first-layer projections P_s, P_d stay fp32 (they are
+//     partial sums of one Linear layer).
 //
 // Organisation (640 threads = 20 warps, one CTA per SM; setmaxnreg moves the
 // control warpgroup's registers to the workers):
@@ -27,6 +32,7 @@
 //     shapes and does bias / gathers, LayerNorm and ReLU in registers.
 #pragma once
 #include <cstdint>
+#include <type_traits>
 #include <cuda_bf16.h>
 #include "ptx.cuh"
 
@@ -74,11 +80,11 @@ struct TileParams {
   const int* key_sorted;      // [E] destination key (== n_nodes for an invalid edge)
   const int* perm;            // [E] input edge id of CSR slot k
   const int* rowptr;          // [N+1]
-  float* e;                   // [E, H] edge state, CSR order (updated in place)
-  float* h;                   // [N, H] node state
+  void* e;                    // [E, H] edge state, CSR order (updated in place); fp32 or bf16
+  void* h;                    // [N, H] node state; fp32 or bf16
   float* ps;                  // [N, H] projections W_s h
   float* pd;                  // [N, H] projections W_d h + b1
-  float* agg;                 // [N, H] row-tiled: sum of incoming messages per node
+  void* agg;                  // [N, H] row-tiled: sum of incoming messages per node; fp32 or bf16
   float* scores;              // [E] input order
   uint32_t* err;              // device error word
 #ifdef GNN_TRACE
@@ -101,31 +107,33 @@ constexpr int kTraceEvents = 512;
 #define GNN_TRACE_W(label) do { } while (0)
 #endif
 
-template <int H>
+template <int H, bool BF>
 struct TileGeom {
   static constexpr int HH = H / 2;                  // columns per worker thread
-  static constexpr int SLOT_COLS = 2 * H;           // D (H cols) + A_hi (H/2) + A_lo (H/2)
+  static constexpr int SLOT_COLS = 2 * H;           // D (H cols) + A_hi (H/2) + A_lo (H/2, fp32 model only)
   static constexpr int TMEM_COLS = 2 * SLOT_COLS;   // two slots: 256 (H=64) or 512 (H=128)
   static constexpr uint32_t PART_BYTES = H * H * 2; // one bf16 H x H matrix part
-  static constexpr uint32_t MAT_BYTES = 2 * PART_BYTES;
-  static constexpr int STAGES = (H == 128) ? 3 : 8; // weight ring depth (matrices)
+  static constexpr uint32_t MAT_BYTES = BF ? PART_BYTES : 2 * PART_BYTES;  // hi [+ lo]
+  static constexpr int STAGES = (192u * 1024u / MAT_BYTES) < 8 ? (192u * 1024u / MAT_BYTES) : 8;  // weight ring depth
   static constexpr uint32_t RING_BYTES = STAGES * MAT_BYTES;
   static constexpr uint32_t IDESC = idesc_bf16_f32(128, H);
+  static constexpr int PRODUCTS = BF ? 1 : 3;       // tcgen05.mma per K step
 };
 
 // Parameter vectors are padded to 16 bytes so the mbarriers after them stay 8-byte aligned.
 __host__ __device__ constexpr int padded_vec_floats(int n) { return (n + 3) & ~3; }
 
-template <int H>
+template <int H, bool BF>
 constexpr uint32_t tile_smem_bytes(int n_vec_floats) {
   // ring (1024-aligned) + vectors + exchange buffers + barriers + alignment slack
-  return TileGeom<H>::RING_BYTES + (uint32_t)padded_vec_floats(n_vec_floats) * 4u + 256 + 1024;
+  return TileGeom<H, BF>::RING_BYTES + (uint32_t)padded_vec_floats(n_vec_floats) * 4u + 256 + 1024;
 }
 
 // ----------------------------------------------------------------- kernel
-template <TileKind KIND, int H>
+template <TileKind KIND, int H, bool BF>
 __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams p) {
-  using G = TileGeom<H>;
+  using G = TileGeom<H, BF>;
+  using SE = typename std::conditional<BF, __nv_bfloat16, float>::type;   // stored state element
   constexpr int NB = H / 8;                          // 8-column blocks per row
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -190,7 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           for (int s = 0; s < 2; ++s) {
             const int tile = 2 * pair + s;
             if (tile >= p.n_tiles) break;
-            if (lane == 0) prefetch_l2_bulk(p.e + (size_t)tile * kTileRows * H, kTileRows * H * 4);
+            if (lane == 0)
+              prefetch_l2_bulk(static_cast<const SE*>(p.e) + (size_t)tile * kTileRows * H, kTileRows * H * sizeof(SE));
 #pragma unroll
             for (int i = 0; i < kTileRows / 32; ++i) {
               const int row = tile * kTileRows + i * 32 + lane;
@@ -254,11 +263,13 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
             for (int ks = 0; ks < H / 16; ++ks) {
               const uint32_t off = (ks >> 2) * (H * 128) + (ks & 3) * 32;
               const uint64_t bh = sdesc_kmajor_sw128(wb + off);
-              const uint64_t bl = sdesc_kmajor_sw128(wb + G::PART_BYTES + off);
+              const uint64_t bl = BF ? 0ull : sdesc_kmajor_sw128(wb + G::PART_BYTES + off);
               const uint32_t acc = (p.job_acc[j] || ks > 0) ? 1u : 0u;
               mma_bf16_ts(d, ahi + ks * 8, bh, G::IDESC, acc);
-              mma_bf16_ts(d, ahi + ks * 8, bl, G::IDESC, 1u);
-              mma_bf16_ts(d, alo + ks * 8, bh, G::IDESC, 1u);
+              if constexpr (!BF) {
+                mma_bf16_ts(d, ahi + ks * 8, bl, G::IDESC, 1u);
+                mma_bf16_ts(d, alo + ks * 8, bh, G::IDESC, 1u);
+              }
             }
             mma_commit(&d_full[s]);
             GNN_TRACE_AT(0, 2 * (int)seq_s[s] + 1 + s * 256);
@@ -328,12 +339,30 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
       return x;
     };
     // Row data keep each thread's four values of a block pair (blocks 2bp and 2bp+1, columns
-    // 2(t%4) and 2(t%4)+1 of each) together, so every row access is one 16-byte vector:
+    // 2(t%4) and 2(t%4)+1 of each) together, so every row access is one 16-byte (fp32) or
+    // 8-byte (bf16) vector:
     //   row-tiled state "T16" (e, h, a): (r, c) at ((r/128)*(H/16) + bp)*2048 + (r%128)*16 + x,
-    //   row-major "RM16" (P_s, P_d):     (r, c) at r*H + bp*16 + x,
+    //   row-major "RM16" (P_s, P_d, fp32): (r, c) at r*H + bp*16 + x,
     // with b = c/8, bp = b/2, x = 4*((c%8)/2) + 2*(b%2) + c%2.
-    auto t16 = [&](const float* base, int row, int bp) -> const float4* {
-      return reinterpret_cast<const float4*>(base + (((size_t)(row >> 7) * (NB / 2) + bp) * 128 + (row & 127)) * 16 + 2 * cq);
+    auto t16 = [&](const void* base, int row, int bp) -> const SE* {
+      return static_cast<const SE*>(base) + (((size_t)(row >> 7) * (NB / 2) + bp) * 128 + (row & 127)) * 16 + 2 * cq;
+    };
+    auto ld_state = [&](const SE* a) -> float4 {
+      if constexpr (BF) {
+        const uint2 u = *reinterpret_cast<const uint2*>(a);
+        const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+        const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+        return make_float4(lo.x, lo.y, hi.x, hi.y);
+      } else {
+        return *reinterpret_cast<const float4*>(a);
+      }
+    };
+    auto st_state = [&](const SE* a, const float4& x) {
+      if constexpr (BF) {
+        *reinterpret_cast<uint2*>(const_cast<SE*>(a)) = make_uint2(pack_bf16x2(x.x, x.y), pack_bf16x2(x.z, x.w));
+      } else {
+        *reinterpret_cast<float4*>(const_cast<SE*>(a)) = x;
+      }
     };
     auto rm16 = [&](const float* base, int row, int bp) -> const float4* {
       return reinterpret_cast<const float4*>(base + (size_t)row * H + bp * 16 + 2 * cq);
@@ -360,14 +389,24 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     // Blocks 4k..4k+3 of both rows (t[4b..4b+3] = block 4k+b: row 0 cols 2(t%4), +1; row 1 the same)
     // -> bf16 hi/lo A operand.  No wait: the caller ends a run of stores with tmem_st_wait().
     auto put_a_chunk = [&](int k, const float* t) {
-      uint32_t hi[8], lo[8];
+      if constexpr (BF) {
+        uint32_t hi[8];
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        split_bf16x2(t[4 * b], t[4 * b + 1], hi[2 * b], lo[2 * b]);
-        split_bf16x2(t[4 * b + 2], t[4 * b + 3], hi[2 * b + 1], lo[2 * b + 1]);
+        for (int b = 0; b < 4; ++b) {
+          hi[2 * b] = pack_bf16x2(t[4 * b], t[4 * b + 1]);
+          hi[2 * b + 1] = pack_bf16x2(t[4 * b + 2], t[4 * b + 3]);
+        }
+        tmem_st_16x128b_x4(ahi_addr + 16 * k, hi);
+      } else {
+        uint32_t hi[8], lo[8];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          split_bf16x2(t[4 * b], t[4 * b + 1], hi[2 * b], lo[2 * b]);
+          split_bf16x2(t[4 * b + 2], t[4 * b + 3], hi[2 * b + 1], lo[2 * b + 1]);
+        }
+        tmem_st_16x128b_x4(ahi_addr + 16 * k, hi);
+        tmem_st_16x128b_x4(alo_addr + 16 * k, lo);
       }
-      tmem_st_16x128b_x4(ahi_addr + 16 * k, hi);
-      tmem_st_16x128b_x4(alo_addr + 16 * k, lo);
     };
     // both rows -> bf16 hi/lo A operand, four blocks per store pair (keeps the
     // temporaries at 16 registers next to the row data)
@@ -390,6 +429,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     // here already has zero mean over the H features: the LayerNorm needs only
     // its variance (the subtraction of the mean is linear and sits in the MMA).
     auto ln_relu = [&](float* v, const float* gamma, const float* beta) {
+      if constexpr (BF) {                      // bf16 weights are not centred: subtract the mean here
+        float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < NB; ++k) { s0 += v[4 * k] + v[4 * k + 1]; s1 += v[4 * k + 2] + v[4 * k + 3]; }
+        const float m0 = quad_sum(s0) * (1.0f / H), m1 = quad_sum(s1) * (1.0f / H);
+#pragma unroll
+        for (int k = 0; k < NB; ++k) { v[4 * k] -= m0; v[4 * k + 1] -= m0; v[4 * k + 2] -= m1; v[4 * k + 3] -= m1; }
+      }
       float q0 = 0.f, q1 = 0.f;
 #pragma unroll
       for (int k = 0; k < NB; ++k) {
@@ -417,7 +464,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     // 4k..4k+3 in the put_a_chunk order.  D stays valid until the slot's next
     // MMA, which this thread has not released yet.
     auto ln_stream = [&](const float* bias, const float* gamma, const float* beta, auto&& emit) {
-      float q0 = 0.f, q1 = 0.f;
+      float q0 = 0.f, q1 = 0.f, s0 = 0.f, s1 = 0.f;
       {
         float t[H / 2];
 #pragma unroll
@@ -432,10 +479,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           const float c2 = t[4 * k + 6] + bb.z, c3 = t[4 * k + 7] + bb.w;
           q0 = fmaf(a0, a0, fmaf(a1, a1, fmaf(a2, a2, fmaf(a3, a3, q0))));
           q1 = fmaf(c0, c0, fmaf(c1, c1, fmaf(c2, c2, fmaf(c3, c3, q1))));
+          if constexpr (BF) { s0 += (a0 + a1) + (a2 + a3); s1 += (c0 + c1) + (c2 + c3); }
         }
       }
-      const float i0 = rsqrtf(quad_sum(q0) * (1.0f / H) + p.eps);
-      const float i1 = rsqrtf(quad_sum(q1) * (1.0f / H) + p.eps);
+      // fp32 model: the host centred the weights, the mean is zero.  bf16 model: one-pass moments.
+      const float m0 = BF ? quad_sum(s0) * (1.0f / H) : 0.f;
+      const float m1 = BF ? quad_sum(s1) * (1.0f / H) : 0.f;
+      const float i0 = rsqrtf(fmaxf(quad_sum(q0) * (1.0f / H) - m0 * m0, 0.f) + p.eps);
+      const float i1 = rsqrtf(fmaxf(quad_sum(q1) * (1.0f / H) - m1 * m1, 0.f) + p.eps);
       float t[2][16];                          // double buffer: chunk k+1 is read while chunk k is emitted
       tmem_ld_16x256b_x4(d_addr, t[0]);
       tmem_ld_wait();
@@ -447,40 +498,40 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         for (int b = 0; b < 4; b += 2) {
           const int kb = 4 * k + b;                        // block index
           const float4 bb = vq4(bias, kb), g = vq4(gamma, kb), be = vq4(beta, kb);
-          u[4 * b] = fmaxf(fmaf((u[4 * b] + bb.x) * i0, g.x, be.x), 0.f);
-          u[4 * b + 1] = fmaxf(fmaf((u[4 * b + 1] + bb.y) * i0, g.y, be.y), 0.f);
-          u[4 * b + 2] = fmaxf(fmaf((u[4 * b + 2] + bb.x) * i1, g.x, be.x), 0.f);
-          u[4 * b + 3] = fmaxf(fmaf((u[4 * b + 3] + bb.y) * i1, g.y, be.y), 0.f);
-          u[4 * b + 4] = fmaxf(fmaf((u[4 * b + 4] + bb.z) * i0, g.z, be.z), 0.f);
-          u[4 * b + 5] = fmaxf(fmaf((u[4 * b + 5] + bb.w) * i0, g.w, be.w), 0.f);
-          u[4 * b + 6] = fmaxf(fmaf((u[4 * b + 6] + bb.z) * i1, g.z, be.z), 0.f);
-          u[4 * b + 7] = fmaxf(fmaf((u[4 * b + 7] + bb.w) * i1, g.w, be.w), 0.f);
+          u[4 * b] = fmaxf(fmaf((u[4 * b] + bb.x - m0) * i0, g.x, be.x), 0.f);
+          u[4 * b + 1] = fmaxf(fmaf((u[4 * b + 1] + bb.y - m0) * i0, g.y, be.y), 0.f);
+          u[4 * b + 2] = fmaxf(fmaf((u[4 * b + 2] + bb.x - m1) * i1, g.x, be.x), 0.f);
+          u[4 * b + 3] = fmaxf(fmaf((u[4 * b + 3] + bb.y - m1) * i1, g.y, be.y), 0.f);
+          u[4 * b + 4] = fmaxf(fmaf((u[4 * b + 4] + bb.z - m0) * i0, g.z, be.z), 0.f);
+          u[4 * b + 5] = fmaxf(fmaf((u[4 * b + 5] + bb.w - m0) * i0, g.w, be.w), 0.f);
+          u[4 * b + 6] = fmaxf(fmaf((u[4 * b + 6] + bb.z - m1) * i1, g.z, be.z), 0.f);
+          u[4 * b + 7] = fmaxf(fmaf((u[4 * b + 7] + bb.w - m1) * i1, g.w, be.w), 0.f);
         }
         emit(k, u);
         if (k + 1 < NB / 4) tmem_ld_wait();
       }
     };
     // blocks 4k..4k+3 of both rows -> row-tiled (T16) output rows
-    auto store_t16_chunk = [&](float* base, int row0, bool ok0, bool ok1, int k, const float* t) {
+    auto store_t16_chunk = [&](void* base, int row0, bool ok0, bool ok1, int k, const float* t) {
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
-        if (ok0) *const_cast<float4*>(t16(base, row0, 2 * k + j)) = get4(t, j, 0);
-        if (ok1) *const_cast<float4*>(t16(base, row0 + 8, 2 * k + j)) = get4(t, j, 1);
+        if (ok0) st_state(t16(base, row0, 2 * k + j), get4(t, j, 0));
+        if (ok1) st_state(t16(base, row0 + 8, 2 * k + j), get4(t, j, 1));
       }
     };
-    auto load_t16 = [&](float* v, const float* base, int row0, bool ok0, bool ok1) {
+    auto load_t16 = [&](float* v, const void* base, int row0, bool ok0, bool ok1) {
       const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
       for (int bp = 0; bp < NB / 2; ++bp) {
-        put4(v, bp, 0, ok0 ? *t16(base, row0, bp) : z);
-        put4(v, bp, 1, ok1 ? *t16(base, row0 + 8, bp) : z);
+        put4(v, bp, 0, ok0 ? ld_state(t16(base, row0, bp)) : z);
+        put4(v, bp, 1, ok1 ? ld_state(t16(base, row0 + 8, bp)) : z);
       }
     };
-    auto store_t16 = [&](float* base, int row0, bool ok0, bool ok1, const float* v) {
+    auto store_t16 = [&](void* base, int row0, bool ok0, bool ok1, const float* v) {
 #pragma unroll
       for (int bp = 0; bp < NB / 2; ++bp) {
-        if (ok0) *const_cast<float4*>(t16(base, row0, bp)) = get4(v, bp, 0);
-        if (ok1) *const_cast<float4*>(t16(base, row0 + 8, bp)) = get4(v, bp, 1);
+        if (ok0) st_state(t16(base, row0, bp), get4(v, bp, 0));
+        if (ok1) st_state(t16(base, row0 + 8, bp), get4(v, bp, 1));
       }
     };
     // D (+ bias) of both rows streamed to a row-major output, 4 blocks per TMEM round trip.
@@ -597,6 +648,10 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           GNN_TRACE_W(11);
         } else {
           const float* wo = vecs + (2 + 3 * (L - 1)) * H;
+          if constexpr (BF) {                  // the head's input is a bf16 activation
+#pragma unroll
+            for (int i = 0; i < 4 * NB; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+          }
           float z0 = 0.f, z1 = 0.f;
 #pragma unroll
           for (int k = 0; k < NB; k += 2) {
@@ -762,17 +817,30 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 template <int H>
 constexpr int agg_nodes_per_block() { return 256 / (H / 4); }
 
-template <int H>
-__global__ void __launch_bounds__(256) aggregate_kernel(const float* __restrict__ e, const int* __restrict__ rowptr,
-                                                        int n_nodes, float* __restrict__ agg) {
+template <int H, bool BF>
+__global__ void __launch_bounds__(256) aggregate_kernel(const void* __restrict__ e_, const int* __restrict__ rowptr,
+                                                        int n_nodes, void* __restrict__ agg_) {
+  using SE = typename std::conditional<BF, __nv_bfloat16, float>::type;
   constexpr int NBP = H / 16;
   constexpr int LPN = H / 4;                         // lanes per node
+  const SE* e = static_cast<const SE*>(e_);
+  SE* agg = static_cast<SE*>(agg_);
   const int li = threadIdx.x % LPN;
   const int bp = li >> 2, q = li & 3;
   const int j = blockIdx.x * agg_nodes_per_block<H>() + (int)threadIdx.x / LPN;
   if (j >= n_nodes) return;
   const int k0 = rowptr[j], k1 = rowptr[j + 1];
-  auto at = [&](int k) { return __ldcs(reinterpret_cast<const float4*>(e + (((size_t)(k >> 7) * NBP + bp) * 128 + (k & 127)) * 16 + 4 * q)); };
+  auto at = [&](int k) -> float4 {
+    const SE* a = e + (((size_t)(k >> 7) * NBP + bp) * 128 + (k & 127)) * 16 + 4 * q;
+    if constexpr (BF) {
+      const uint2 u = __ldcs(reinterpret_cast<const uint2*>(a));
+      const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+      const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+      return make_float4(lo.x, lo.y, hi.x, hi.y);
+    } else {
+      return __ldcs(reinterpret_cast<const float4*>(a));
+    }
+  };
   float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
   int k = k0;
   for (; k + 4 <= k1; k += 4) {
@@ -786,7 +854,12 @@ __global__ void __launch_bounds__(256) aggregate_kernel(const float* __restrict_
     const float4 x = at(k);
     a.x += x.x; a.y += x.y; a.z += x.z; a.w += x.w;
   }
-  *reinterpret_cast<float4*>(agg + (((size_t)(j >> 7) * NBP + bp) * 128 + (j & 127)) * 16 + 4 * q) = a;
+  SE* out = agg + (((size_t)(j >> 7) * NBP + bp) * 128 + (j & 127)) * 16 + 4 * q;
+  if constexpr (BF) {                                // the aggregate is a bf16 activation
+    *reinterpret_cast<uint2*>(out) = make_uint2(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w));
+  } else {
+    *reinterpret_cast<float4*>(out) = a;
+  }
 }
 
 }  // namespace gnn

@@ -145,9 +145,12 @@ def _hand_model():
     return W
 
 
-def _hand_forward(W, x, src, dst, T):
+def _hand_forward(W, x, src, dst, T, rnd=None):
+    """Scalar forward of the hand model; `rnd` (if given) rounds every layer output and the
+    aggregate, as the bf16 model does."""
     f32 = np.float32
     n, E = x.shape[0], len(src)
+    r = rnd if rnd is not None else (lambda t: t)
 
     def lin(Wb, z):
         Wm, b = Wb
@@ -156,7 +159,8 @@ def _hand_forward(W, x, src, dst, T):
     def layer(params, z):
         Wm, b, g, bt = params[0]
         v = lin((Wm, b), z)
-        return _relu2(_ln2(v[0], v[1], g, bt))
+        o = _relu2(_ln2(v[0], v[1], g, bt))
+        return (r(o[0]), r(o[1]))
 
     h = [layer(W["node_encoder"], [float(x[j][0]), float(x[j][1])]) for j in range(n)]
     e = []
@@ -172,6 +176,7 @@ def _hand_forward(W, x, src, dst, T):
         a = [[0.0, 0.0] for _ in range(n)]
         for k in range(E):
             a[dst[k]][0] += m[k][0]; a[dst[k]][1] += m[k][1]
+        a = [[r(a[j][0]), r(a[j][1])] for j in range(n)]
         h = [layer(W["node_network"], list(h[j]) + a[j]) for j in range(n)]
     logits = []
     for k in range(E):
@@ -298,8 +303,8 @@ def _mutants():
         var = ((v - mu) ** 2).sum(-1, keepdims=True) / max(v.shape[-1] - 1, 1)
         return g * (v - mu) / np.sqrt(var + eps) + b
 
-    def agg_twice(m, dst, n):
-        return 2 * agg(m, dst, n)
+    def agg_twice(m, dst, n, dtype=np.float64):
+        return 2 * agg(m, dst, n, dtype)
 
     def ef_neg(x, s, d):
         return -ef(x, s, d)
@@ -320,3 +325,47 @@ def test_worked_example_kills_planted_mistakes(name, monkeypatch):
     monkeypatch.setattr(O, attr, fn)
     _, got = O.forward(W, HAND_X, HAND_EI, 2, HAND_EPS, return_logits=True)
     assert np.abs(got - want).max() > 1e-6, name
+
+
+# ------------------------------------------------------------- bf16 model
+
+def _bf16_scalar(t: float) -> float:
+    """Nearest bfloat16 of a Python float: t = m * 2**e with 0.5 <= |m| < 1, keep 8
+    significant bits; Python's round() takes halfway cases to even."""
+    if t == 0.0:
+        return 0.0
+    m, e = math.frexp(t)
+    return math.ldexp(round(m * 256), e - 8)
+
+
+def test_round_bf16_values():
+    # spacing next to 1 is 2^-7; exact halfway cases go to the even neighbour
+    cases = {1.0: 1.0, 1.0 + 2 ** -8: 1.0, 1.0 + 3 * 2 ** -8: 1.0 + 2 ** -6, 1.0 + 2 ** -7: 1.0 + 2 ** -7,
+             0.1: 0.10009765625, -2.5: -2.5, 255.5: 256.0, 257.0: 256.0, 3.0e-3: 0.0030059814453125}
+    got = O.round_bf16(np.array(list(cases)))
+    np.testing.assert_array_equal(got, list(cases.values()))
+    # agrees with an independent bit-level rounding of float32 values
+    v = np.random.default_rng(3).standard_normal(20000).astype(np.float32) * 7
+    np.testing.assert_array_equal(O.round_bf16(v.astype(np.float64)), S._round_bf16(v).astype(np.float64))
+    assert all(O.round_bf16(np.array([t]))[0] == _bf16_scalar(t) for t in v[:500].tolist())
+
+
+@pytest.mark.parametrize("T", [1, 2])
+def test_bf16_worked_example(T):
+    """The bf16 model rounds every layer output and the aggregate, nothing else."""
+    W = _hand_model()
+    _, got = O.forward(W, HAND_X, HAND_EI, T, HAND_EPS, return_logits=True, bf16=True)
+    want = _hand_forward(W, HAND_X, HAND_EI[0].tolist(), HAND_EI[1].tolist(), T, rnd=_bf16_scalar)
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+    plain = _hand_forward(W, HAND_X, HAND_EI[0].tolist(), HAND_EI[1].tolist(), T)
+    assert np.abs(np.array(want) - np.array(plain)).max() > 1e-4      # the rounding points are live
+
+
+def test_bf16_model_close_to_unrounded_model():
+    cfg = S.ModelConfig(3, 2, 64, 2, 2, S.PRECISION_BF16)
+    W = S.init_weights(cfg, 4)
+    x, ei = S.random_graph(60, 300, 3, 2)
+    _, z64 = O.forward(W, x, ei, cfg.n_iters, return_logits=True)
+    _, zb = O.forward(W, x, ei, cfg.n_iters, return_logits=True, bf16=True)
+    d = np.abs(zb - z64)
+    assert 1e-4 < d.max() < 0.5 and d.mean() < 0.05
