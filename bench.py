@@ -70,7 +70,8 @@ def step_model(w: S.Workload):
 
 
 # ------------------------------------------------------------------ ncu traffic
-PROFILE_FOR_KERNEL = {"edge_update": "edge_update_full_event.md"}
+PROFILE_FOR_KERNEL = {("edge_update", False): "edge_update_full_event.md",
+                      ("edge_update", True): "edge_update_bf16_full_event.md"}
 KERNEL_SOURCES = ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh", "gnn_api.cu")
 
 
@@ -88,10 +89,10 @@ def source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel: str):
-    """DRAM bytes per launch from the committed ncu summary of `kernel`, or None when there is
-    none or the kernel sources changed since the counters were taken."""
-    name = PROFILE_FOR_KERNEL.get(kernel)
+def profiled_traffic(kernel: str, bf16: bool = False):
+    """DRAM bytes per launch from the committed ncu summary of `kernel` (fp32 or bf16 model), or
+    None when there is none or the kernel sources changed since the counters were taken."""
+    name = PROFILE_FOR_KERNEL.get((kernel, bf16))
     path = os.path.join(ROOT, "profiles", name) if name else None
     if not path or not os.path.exists(path):
         return None
@@ -335,7 +336,7 @@ def run_gb300(args, rank: int, world: int, local: int):
     if dom_model is not None:
         achieved = dom_model["bytes"] / dom_avg_s / 1e9
         roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"],
-                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": profiled_traffic(dom),
+                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": profiled_traffic(dom, w.model.precision == S.PRECISION_BF16),
                     "peak_source": f"{peak_src} (hbm_gbs, copy burst) -- of {peak_src}",
                     "bytes_per_launch": dom_model["bytes"], "avg_launch_ms": dom_avg_s * 1e3,
                     "tensor_tflops_executed": (1 if w.model.precision == S.PRECISION_BF16 else 3)
