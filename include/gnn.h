@@ -132,6 +132,27 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
                    int64_t n_edges, float* edge_scores, gnn_stream_t stream);
 
 /*
+ * gnn_track_labels -- track candidates from scored edges: one integer label per hit.  The
+ * edge-classification scores are thresholded and the weakly connected components of the kept
+ * edges are the track candidates (paper Section 2.1, the step after the interaction network);
+ * the service returns an integer label per space point (Section 2.3).
+ *
+ *   edge_scores device float32 [n_edges], input edge order (as gnn_infer writes them)
+ *   edge_index  device int32 [2, n_edges]: row 0 sources, row 1 destinations
+ *   threshold   an edge is kept when its score is > threshold (NaN scores are never kept)
+ *   labels      device int32 [n_nodes], output: the smallest node id of the hit's component
+ *               (a hit without kept edges is its own component); caller-owned
+ *
+ * Edges with an endpoint outside [0, n_nodes) are skipped.  The labels do not depend on thread
+ * or edge order.  Enqueued on `stream`; uses no workspace (the labels array is the union-find
+ * forest).  A union retry loop that never settles records GNN_ERR_DEVICE_TIMEOUT in the context's
+ * device error word (see gnn_status).  Errors: INVALID_ARG (null pointer, negative or too large
+ * sizes, n_nodes == 0 with edges), CUDA.
+ */
+int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge_index, int64_t n_nodes,
+                     int64_t n_edges, float threshold, int32_t* labels, gnn_stream_t stream);
+
+/*
  * gnn_profile_enable -- when on != 0, later gnn_infer / gnn_infer_host calls
  * record a CUDA event pair on their stream around every kernel group, so
  * gnn_profile_read can report device time per group.  Off by default.

@@ -157,3 +157,28 @@ def forward(weights: dict, x: np.ndarray, edge_index: np.ndarray, n_iters: int,
     if return_states:
         out.append({"h": h, "e": e})
     return out[0] if len(out) == 1 else tuple(out)
+
+
+def track_labels(scores: np.ndarray, edge_index: np.ndarray, n_nodes: int, threshold: float = 0.5) -> np.ndarray:
+    """Track candidates (Section 2.1: the edge scores are thresholded and the weakly connected
+    components of the kept edges are the tracks; Section 2.3: one integer label per space point).
+
+    An edge is kept when its score is > threshold (NaN is never kept) and both endpoints lie in
+    [0, n_nodes).  Each hit is labelled by the smallest node id of its component, found by
+    repeating  label[u] = label[v] = min(label[u], label[v])  over the kept edges until no label
+    changes (labels only decrease, and the smallest id of a component reaches every member)."""
+    s = np.asarray(scores, dtype=np.float64)
+    u = np.asarray(edge_index[0], dtype=np.int64)
+    v = np.asarray(edge_index[1], dtype=np.int64)
+    keep = (s > threshold) & (u >= 0) & (u < n_nodes) & (v >= 0) & (v < n_nodes)
+    u, v = u[keep], v[keep]
+    label = np.arange(n_nodes, dtype=np.int64)
+    while True:
+        m = np.minimum(label[u], label[v])
+        new = label.copy()
+        np.minimum.at(new, u, m)
+        np.minimum.at(new, v, m)
+        if np.array_equal(new, label):
+            return label.astype(np.int32)
+        label = new
+

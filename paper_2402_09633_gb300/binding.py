@@ -16,7 +16,7 @@ ERRORS = {-1: "INVALID_ARG", -2: "BAD_WEIGHTS", -3: "OOM", -4: "CUDA", -5: "INDE
           -6: "DEVICE_TIMEOUT"}
 EXPORTED = ("gnn_create", "gnn_reserve", "gnn_infer", "gnn_infer_host", "gnn_status",
             "gnn_destroy", "gnn_error_string", "gnn_debug_copy", "gnn_profile_enable",
-            "gnn_profile_read")
+            "gnn_profile_read", "gnn_track_labels", "gnn_csr_build_noalloc")
 PROFILE_GROUPS = ("csr_build", "node_encoder", "edge_encoder", "edge_update", "node_update",
                   "classifier", "host_copies", "aggregate")
 
@@ -63,6 +63,8 @@ def load_library(path: str = LIB_PATH):
     lib.gnn_profile_enable.restype = i32
     lib.gnn_profile_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64), i32]
     lib.gnn_profile_read.restype = i32
+    lib.gnn_track_labels.argtypes = [vp, vp, vp, i64, i64, ctypes.c_float, vp, vp]
+    lib.gnn_track_labels.restype = i32
     _lib = lib
     return lib
 
@@ -124,6 +126,23 @@ class InteractionNetwork:
         if rc not in (GNN_OK, -5):
             raise GnnError(rc, "gnn_infer_host")
         return rc
+
+    def track_labels(self, scores, edge_index, n_nodes: int, threshold: float = 0.5, labels=None,
+                     stream=None):
+        """Track candidates: int32 [n_nodes] cuda labels (smallest hit id of each connected
+        component of the edges with score > threshold)."""
+        import torch
+        assert scores.is_cuda and scores.dtype == torch.float32 and scores.is_contiguous()
+        assert edge_index.is_cuda and edge_index.dtype == torch.int32 and edge_index.is_contiguous()
+        if labels is None:
+            labels = torch.empty(n_nodes, dtype=torch.int32, device=scores.device)
+        rc = self.lib.gnn_track_labels(self.handle, ctypes.c_void_p(scores.data_ptr()),
+                                       ctypes.c_void_p(edge_index.data_ptr()), n_nodes, edge_index.shape[1],
+                                       float(threshold), ctypes.c_void_p(labels.data_ptr()),
+                                       _stream_handle(stream))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_track_labels")
+        return labels
 
     def profile(self, on: bool = True):
         self.lib.gnn_profile_enable(self.handle, 1 if on else 0)

@@ -1,0 +1,74 @@
+// Track candidates from scored edges: weakly connected components of the edges
+// whose score passes a threshold, labelled by the smallest hit id in each
+// component (one integer label per space point).
+//
+// Lock-free union-find on the label array itself (no scratch): every link
+// hangs the larger root under the smaller one, so parent[v] <= v always holds
+// and each component's final root is its smallest member.  That makes the
+// labels canonical: independent of thread order and of the order of the
+// edges.  During the unions, path halving writes are plain stores; they race
+// benignly because every value written is an ancestor of the node.  The final
+// pass only reads the forest (see cc_flatten_kernel).
+#pragma once
+#include <cstdint>
+#include "ptx.cuh"
+
+namespace gnn {
+
+constexpr uint32_t kUnionRetryLimit = 1u << 24;   // a retry loop that long records DEV_ERR_TIMEOUT
+
+__global__ void cc_init_kernel(int32_t* parent, int n) {
+  const int v = blockIdx.x * blockDim.x + threadIdx.x;
+  if (v < n) parent[v] = v;
+}
+
+__device__ __forceinline__ int cc_find(int32_t* parent, int x) {
+  volatile int32_t* p = parent;
+  for (uint32_t it = 0; it < kUnionRetryLimit; ++it) {
+    const int px = p[x];
+    if (px == x) return x;
+    const int gx = p[px];
+    if (gx != px) p[x] = gx;                           // path halving
+    x = px;
+  }
+  return x;
+}
+
+// One thread per edge: unite the endpoints of every edge kept by the threshold.  Edges with an
+// endpoint outside [0, n) and edges whose score is NaN or <= threshold are skipped.
+__global__ void cc_union_kernel(const float* __restrict__ scores, const int32_t* __restrict__ ei, int n, int m,
+                                float threshold, int32_t* parent, uint32_t* err) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= m) return;
+  const float s = scores[k];
+  if (!(s > threshold)) return;
+  int u = ei[k], v = ei[(size_t)m + k];
+  if (u < 0 || u >= n || v < 0 || v >= n) return;
+  for (uint32_t it = 0;; ++it) {
+    if (it == kUnionRetryLimit) { atomicOr(err, DEV_ERR_TIMEOUT); return; }
+    u = cc_find(parent, u);
+    v = cc_find(parent, v);
+    if (u == v) return;
+    if (u < v) { const int t = u; u = v; v = t; }     // u: the larger root, hung under v
+    if (atomicCAS(parent + u, u, v) == u) return;
+  }
+}
+
+// labels[v] = root of v (the smallest id of its component).  The walk only reads: a path-halving
+// store from another thread could otherwise land on parent[v] after v has written its root and
+// leave v pointing at an intermediate ancestor.  Every value a reader meets is an ancestor (an
+// old parent or a final root), so each walk still ends at its root.
+__global__ void cc_flatten_kernel(int32_t* parent, int n) {
+  const int v = blockIdx.x * blockDim.x + threadIdx.x;
+  if (v >= n) return;
+  volatile int32_t* p = parent;
+  int x = v;
+  for (uint32_t it = 0; it < kUnionRetryLimit; ++it) {
+    const int px = p[x];
+    if (px == x) break;
+    x = px;
+  }
+  parent[v] = x;
+}
+
+}  // namespace gnn

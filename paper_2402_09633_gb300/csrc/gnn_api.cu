@@ -23,6 +23,7 @@
 #include <vector>
 
 #include "../../include/gnn.h"
+#include "components.cuh"
 #include "csr.cuh"
 #include "mlp_tiles.cuh"
 
@@ -563,6 +564,20 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
   prof_end(ctx, pr, st);
   if (err != cudaSuccess) return cuda_fail(err);
   return gnn_status(ctx, stream);
+}
+
+int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge_index, int64_t n_nodes,
+                     int64_t n_edges, float threshold, int32_t* labels, gnn_stream_t stream) {
+  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX) return GNN_ERR_INVALID_ARG;
+  if (n_nodes == 0) return n_edges == 0 ? GNN_OK : GNN_ERR_INVALID_ARG;
+  if (!labels || (n_edges > 0 && (!edge_scores || !edge_index))) return GNN_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  const int N = (int)n_nodes, E = (int)n_edges, tb = 256;
+  cc_init_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
+  if (E > 0) cc_union_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(edge_scores, edge_index, N, E, threshold, labels, ctx->d_err);
+  cc_flatten_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
 
 #ifdef GNN_TRACE

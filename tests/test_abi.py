@@ -45,6 +45,9 @@ def test_invalid_arguments_rejected_on_host():
     assert lib.gnn_create(None, None, 0, ctypes.byref(h)) == -1
     assert lib.gnn_infer(None, None, None, 0, 0, None, None) == -1
     assert lib.gnn_reserve(None, 1, 1) == -1
+    lib.gnn_track_labels.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                                     ctypes.c_int64, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p]
+    assert lib.gnn_track_labels(None, None, None, 5, 3, 0.5, None, None) == -1
 
 
 def test_python_path_fails_loudly_without_library(tmp_path):

@@ -369,3 +369,60 @@ def test_bf16_model_close_to_unrounded_model():
     _, zb = O.forward(W, x, ei, cfg.n_iters, return_logits=True, bf16=True)
     d = np.abs(zb - z64)
     assert 1e-4 < d.max() < 0.5 and d.mean() < 0.05
+
+
+# ------------------------------------------------------------- track labels
+
+def _bfs_labels(edges, n):
+    """Brute force: breadth-first search from every unvisited node in increasing id order."""
+    adj = [[] for _ in range(n)]
+    for a, b in edges:
+        adj[a].append(b); adj[b].append(a)
+    lab = [-1] * n
+    for s0 in range(n):
+        if lab[s0] >= 0:
+            continue
+        lab[s0] = s0
+        todo = [s0]
+        while todo:
+            x = todo.pop()
+            for y in adj[x]:
+                if lab[y] < 0:
+                    lab[y] = s0; todo.append(y)
+    return lab
+
+
+def test_track_labels_against_breadth_first_search():
+    rng = np.random.default_rng(8)
+    for n, m in [(1, 0), (5, 3), (40, 30), (300, 250), (300, 900)]:
+        ei = rng.integers(0, n, size=(2, m)).astype(np.int32)
+        sc = rng.random(m)
+        for thr in (0.0, 0.5, 0.9):
+            kept = [(int(a), int(b)) for a, b, x in zip(ei[0], ei[1], sc) if x > thr]
+            assert O.track_labels(sc, ei, n, thr).tolist() == _bfs_labels(kept, n)
+
+
+def test_track_labels_special_cases():
+    ei = np.array([[0, 1, 3, 4, 2], [1, 2, 3, 9, 7]], np.int32)    # self-loop, out-of-range endpoints
+    sc = np.array([0.9, 0.9, 0.9, 0.9, np.nan])
+    assert O.track_labels(sc, ei, 6, 0.5).tolist() == [0, 0, 0, 3, 4, 5]
+    assert O.track_labels(sc, ei, 6, 0.95).tolist() == [0, 1, 2, 3, 4, 5]   # nothing kept
+    assert O.track_labels(np.zeros(0), np.zeros((2, 0), np.int32), 3).tolist() == [0, 1, 2]
+    # a path given leaves-first still labels every hit with the smallest id
+    ei = np.array([[5, 4, 3, 2, 1], [4, 3, 2, 1, 0]], np.int32)
+    assert O.track_labels(np.ones(5), ei, 6).tolist() == [0] * 6
+
+
+def test_track_labels_against_library_components():
+    sp = pytest.importorskip("scipy.sparse")
+    csg = pytest.importorskip("scipy.sparse.csgraph")
+    rng = np.random.default_rng(9)
+    n, m = 5000, 4000
+    ei = rng.integers(0, n, size=(2, m)).astype(np.int32)
+    sc = rng.random(m)
+    keep = sc > 0.3
+    g = sp.coo_matrix((np.ones(keep.sum()), (ei[0][keep], ei[1][keep])), shape=(n, n))
+    _, comp = csg.connected_components(g, directed=True, connection="weak")
+    smallest = np.full(comp.max() + 1, n)
+    np.minimum.at(smallest, comp, np.arange(n))
+    np.testing.assert_array_equal(O.track_labels(sc, ei, n, 0.3), smallest[comp])
