@@ -195,6 +195,22 @@ const char* gnn_error_string(int code);
 int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_t stream);
 
 /*
+ * Failure-injection hooks for tests (no paper counterpart).  Neither faults nor hangs a GPU.
+ *
+ * gnn_debug_fail_allocs -- the next n device allocations made by the library (context creation,
+ * workspace growth, gnn_infer_host staging) fail as if the device were out of memory, so the
+ * GNN_ERR_OOM paths can be exercised; n = 0 cancels.  Process-wide.  Errors: INVALID_ARG (n < 0).
+ *
+ * gnn_debug_wait_timeout -- enqueue on `stream` one kernel that waits, through the same bounded
+ * wait every pipeline wait in the library uses, on an mbarrier that nothing completes; after
+ * limit_ns nanoseconds (0 < limit_ns <= 2e9) the wait gives up and records GNN_ERR_DEVICE_TIMEOUT
+ * in the context's device error word, which gnn_status then returns (and clears).  The context
+ * stays usable.  Errors: INVALID_ARG, CUDA.
+ */
+int gnn_debug_fail_allocs(int n);
+int gnn_debug_wait_timeout(gnn_ctx* ctx, int64_t limit_ns, gnn_stream_t stream);
+
+/*
  * gnn_csr_build_noalloc -- the destination-keyed CSR of an edge list, built
  * without allocating any device memory.  (Library plumbing: the paper has no
  * counterpart.)  It is for callers that must not allocate: a serving backend

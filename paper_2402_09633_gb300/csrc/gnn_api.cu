@@ -15,6 +15,7 @@
 // update, node update with aggregation + projections) -> classifier.
 #include <cuda_runtime.h>
 #include <algorithm>
+#include <atomic>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -124,6 +125,32 @@ void pack_block(const float* W, int ld, int col0, int H, bool with_lo, uint8_t* 
 }
 
 void push(std::vector<float>& v, const float* p, size_t n) { v.insert(v.end(), p, p + n); }
+
+// Test hook: the next g_fail_allocs device allocations made by the library fail (host-side fault
+// injection for the allocation-failure paths; see gnn_debug_fail_allocs).
+std::atomic<int> g_fail_allocs{0};
+
+cudaError_t dev_alloc(void** p, size_t bytes) {
+  int n = g_fail_allocs.load();
+  while (n > 0 && !g_fail_allocs.compare_exchange_weak(n, n - 1)) {
+  }
+  if (n > 0) {
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  return cudaMalloc(p, bytes);
+}
+
+// A kernel that waits, through the library's bounded wait, on an mbarrier nothing arrives on.
+__global__ void wait_timeout_kernel(uint64_t limit_ns, uint32_t* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  abort_flag = 0;
+  fence_mbar_init();
+  bounded_wait(&bar, 0, &abort_flag, err, limit_ns);
+}
 
 int cuda_fail(cudaError_t e) {
   (void)cudaGetLastError();
@@ -250,7 +277,7 @@ int ensure_workspace(gnn_ctx* c, int64_t N, int64_t E) {
                         al(se * e_pad * H) + 2 * al(se * n_pad * H) + 2 * al(4 * n * H);
   free_workspace(c);
   void* ws = nullptr;
-  cudaError_t err = cudaMalloc(&ws, (size_t)total);
+  cudaError_t err = dev_alloc(&ws, (size_t)total);
   if (err != cudaSuccess) return cuda_fail(err);
   c->ws = ws;
   uint8_t* q = (uint8_t*)ws;
@@ -484,10 +511,10 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     }
     v.resize(padded_vec_floats((int)v.size()), 0.f);
   }
-  err = cudaMalloc(&c->d_mats, packed.size());
+  err = dev_alloc((void**)&c->d_mats, packed.size());
   if (err == cudaSuccess) err = cudaMemcpy(c->d_mats, packed.data(), packed.size(), cudaMemcpyHostToDevice);
   for (int i = 0; i < 7 && err == cudaSuccess; ++i) {
-    err = cudaMalloc(&c->plan[i].d_vecs, c->plan[i].vecs.size() * 4);
+    err = dev_alloc((void**)&c->plan[i].d_vecs, c->plan[i].vecs.size() * 4);
     if (err == cudaSuccess)
       err = cudaMemcpy(c->plan[i].d_vecs, c->plan[i].vecs.data(), c->plan[i].vecs.size() * 4, cudaMemcpyHostToDevice);
   }
@@ -496,7 +523,7 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
   if (err == cudaSuccess) err = cudaMemset(c->trace, 0, 3 * kTraceEvents * 8);
   if (const char* k = getenv("GNN_TRACE_KIND")) c->trace_kind = atoi(k);
 #endif
-  if (err == cudaSuccess) err = cudaMalloc(&c->d_err, 4);
+  if (err == cudaSuccess) err = dev_alloc((void**)&c->d_err, 4);
   if (err == cudaSuccess) err = cudaMemset(c->d_err, 0, 4);
   if (err != cudaSuccess) { gnn_destroy(c); return cuda_fail(err); }
   *out = c;
@@ -544,7 +571,7 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
   const size_t need = al(bx) + al(be) + al(bs);
   if (need > ctx->stage_bytes) {
     if (ctx->stage) { cudaStreamSynchronize(st); cudaFree(ctx->stage); ctx->stage = nullptr; ctx->stage_bytes = 0; }
-    const cudaError_t err = cudaMalloc(&ctx->stage, need);
+    const cudaError_t err = dev_alloc(&ctx->stage, need);
     if (err != cudaSuccess) return cuda_fail(err);
     ctx->stage_bytes = need;
   }
@@ -586,6 +613,19 @@ int gnn_trace_read(gnn_ctx* ctx, unsigned long long* host) {
   return cudaMemcpy(host, ctx->trace, 3 * kTraceEvents * 8, cudaMemcpyDeviceToHost) == cudaSuccess ? 0 : -4;
 }
 #endif
+
+int gnn_debug_fail_allocs(int n) {
+  if (n < 0) return GNN_ERR_INVALID_ARG;
+  g_fail_allocs.store(n);
+  return GNN_OK;
+}
+
+int gnn_debug_wait_timeout(gnn_ctx* ctx, int64_t limit_ns, gnn_stream_t stream) {
+  if (!ctx || limit_ns <= 0 || limit_ns > (int64_t)kWaitLimitNs) return GNN_ERR_INVALID_ARG;
+  wait_timeout_kernel<<<1, 32, 0, (cudaStream_t)stream>>>((uint64_t)limit_ns, ctx->d_err);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
 
 int gnn_profile_enable(gnn_ctx* ctx, int on) {
   if (!ctx) return GNN_ERR_INVALID_ARG;

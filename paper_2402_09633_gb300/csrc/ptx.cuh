@@ -72,16 +72,16 @@ __device__ __forceinline__ uint32_t atomic_add_acq_rel_shared(uint32_t* addr, ui
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
 
 // Waits until the mbarrier phase with `parity` completed, or until `*abort`
-// becomes non-zero, or until the limit expires (then records DEV_ERR_TIMEOUT
+// becomes non-zero, or until `limit_ns` expires (then records DEV_ERR_TIMEOUT
 // in *err and sets *abort).  Returns true when the phase completed.
-__device__ __forceinline__ bool bounded_wait(uint64_t* bar, uint32_t parity,
-                                             volatile int* abort, uint32_t* err) {
+__device__ __forceinline__ bool bounded_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* err,
+                                             uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if ((it & 63u) == 63u && global_timer_ns() - t0 > kWaitLimitNs) {
+    if ((it & 63u) == 63u && global_timer_ns() - t0 > limit_ns) {
       atomicOr(err, DEV_ERR_TIMEOUT);
       *abort = 1;
       return false;
