@@ -132,6 +132,37 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
                    int64_t n_edges, float* edge_scores, gnn_stream_t stream);
 
 /*
+ * gnn_filter_load -- load the filtering MLP (paper Section 2.1: the step before the GNN scores every
+ * candidate edge from the raw features of its two hits; applyFiltering then drops the edges below
+ * a fixed threshold).  Network: s = sigmoid(w_o . MLP_L([x_src, x_dst]) + b_o), each of its L
+ * layers Linear -> LayerNorm -> ReLU, in the context's precision and hidden width.
+ * Blob (little-endian, copied; the caller may free it): eight int32 (magic 0x4C464E47 "GNFL",
+ * version 1, n_node_feat, hidden, mlp_layers (2..4), precision, two reserved), float32 ln_eps,
+ * int32 reserved, int64 float count, then float32 arrays: per layer W [H, in] row-major, b, gamma,
+ * beta (in = 2 * n_node_feat for layer 1, H afterwards), then w_o [H], b_o [1].  n_node_feat,
+ * hidden and precision must equal the context's.  A later call replaces the filter.
+ * Errors: INVALID_ARG, BAD_WEIGHTS, OOM, CUDA.  Synchronous.
+ *
+ * gnn_filter_edges -- score every candidate edge with the filtering MLP and keep those with
+ * score > threshold, in input order.
+ *   node_feats  device float32 [n_nodes, n_node_feat]
+ *   edge_index  device int32 [2, n_edges] (row 0 sources, row 1 destinations)
+ *   edge_scores device float32 [n_edges], output: filter score of every input edge (NaN for an edge
+ *               with an endpoint out of range, which is never kept; gnn_status then reports
+ *               INDEX_RANGE)
+ *   kept_index  device int32 with room for [2, n_edges], output: the kept edges as a contiguous
+ *               [2, n_kept] edge index (row 1 starts at n_kept), ready for gnn_infer
+ *   kept_id     device int32 [n_edges] or NULL, output: input id of every kept edge
+ *   n_kept      device int32 [1], output
+ * All buffers are caller-owned.  Enqueued on `stream`; uses the context's workspace (it may grow,
+ * as in gnn_infer).  Errors: INVALID_ARG (no filter loaded, null pointer, bad sizes), OOM, CUDA.
+ */
+int gnn_filter_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes);
+int gnn_filter_edges(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
+                     int64_t n_edges, float threshold, float* edge_scores, int32_t* kept_index, int32_t* kept_id,
+                     int32_t* n_kept, gnn_stream_t stream);
+
+/*
  * gnn_track_labels -- track candidates from scored edges: one integer label per hit.  The
  * edge-classification scores are thresholded and the weakly connected components of the kept
  * edges are the track candidates (paper Section 2.1, the step after the interaction network);
@@ -162,8 +193,8 @@ int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge
  * kernel launches launches[g]; then clear the records.  Groups: 0 CSR build
  * (all its kernels), 1 node encoder, 2 edge encoder, 3 edge update, 4 node
  * update, 5 classifier, 6 host<->device copies of gnn_infer_host, 7 message
- * aggregation.  Either output pointer may be NULL.  Returns the number of
- * groups (8) or an error.
+ * aggregation, 8 filtering MLP.  Either output pointer may be NULL.  Returns
+ * the number of groups (9) or an error.
  */
 int gnn_profile_enable(gnn_ctx* ctx, int on);
 int gnn_profile_read(gnn_ctx* ctx, double* ms, int64_t* launches, int n_groups);

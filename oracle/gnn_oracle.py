@@ -182,3 +182,32 @@ def track_labels(scores: np.ndarray, edge_index: np.ndarray, n_nodes: int, thres
             return label.astype(np.int32)
         label = new
 
+
+def filter_scores(fw: dict, x: np.ndarray, edge_index: np.ndarray, eps: float = 1e-5, bf16: bool = False,
+                  return_logits: bool = False):
+    """Filtering step (Section 2.1: before the GNN, an MLP scores every candidate edge from the raw
+    features of its two hits): s = sigmoid(w_o . MLP([x_src, x_dst]) + b_o).  `fw` holds 'layers'
+    [(W, b, gamma, beta)], 'head_w' [H], 'head_b' [1].  Edges with an endpoint outside
+    [0, N) score NaN.  `bf16` rounds every layer output to bfloat16, as in forward()."""
+    x = np.asarray(x, dtype=np.float32)
+    src = np.asarray(edge_index[0], dtype=np.int64)
+    dst = np.asarray(edge_index[1], dtype=np.int64)
+    n = x.shape[0]
+    ok = (src >= 0) & (src < n) & (dst >= 0) & (dst < n)
+    s_, d_ = np.where(ok, src, 0), np.where(ok, dst, 0)
+    v = np.concatenate([x[s_], x[d_]], axis=1).astype(np.float64)
+    c = mlp(v, fw["layers"], eps, round_bf16 if bf16 else None)
+    logits = c @ np.asarray(fw["head_w"], np.float64) + float(np.asarray(fw["head_b"])[0])
+    logits = np.where(ok, logits, np.nan)
+    scores = sigmoid(np.where(ok, logits, 0.0))
+    scores = np.where(ok, scores, np.nan)
+    return (scores, logits) if return_logits else scores
+
+
+def apply_filtering(scores: np.ndarray, edge_index: np.ndarray, threshold: float):
+    """applyFiltering (Section 2.1): the edges whose score is > threshold (NaN never), in input
+    order.  Returns (kept edge index [2, n_kept], input ids of the kept edges)."""
+    keep = np.asarray(scores) > threshold
+    ids = np.nonzero(keep)[0]
+    return np.asarray(edge_index)[:, ids], ids
+

@@ -16,9 +16,10 @@ ERRORS = {-1: "INVALID_ARG", -2: "BAD_WEIGHTS", -3: "OOM", -4: "CUDA", -5: "INDE
           -6: "DEVICE_TIMEOUT"}
 EXPORTED = ("gnn_create", "gnn_reserve", "gnn_infer", "gnn_infer_host", "gnn_status",
             "gnn_destroy", "gnn_error_string", "gnn_debug_copy", "gnn_profile_enable",
-            "gnn_profile_read", "gnn_track_labels", "gnn_csr_build_noalloc")
+            "gnn_profile_read", "gnn_track_labels", "gnn_csr_build_noalloc", "gnn_filter_load",
+            "gnn_filter_edges")
 PROFILE_GROUPS = ("csr_build", "node_encoder", "edge_encoder", "edge_update", "node_update",
-                  "classifier", "host_copies", "aggregate")
+                  "classifier", "host_copies", "aggregate", "filter")
 
 
 class GnnError(RuntimeError):
@@ -65,6 +66,10 @@ def load_library(path: str = LIB_PATH):
     lib.gnn_profile_read.restype = i32
     lib.gnn_track_labels.argtypes = [vp, vp, vp, i64, i64, ctypes.c_float, vp, vp]
     lib.gnn_track_labels.restype = i32
+    lib.gnn_filter_load.argtypes = [vp, vp, ctypes.c_size_t]
+    lib.gnn_filter_load.restype = i32
+    lib.gnn_filter_edges.argtypes = [vp, vp, vp, i64, i64, ctypes.c_float, vp, vp, vp, vp, vp]
+    lib.gnn_filter_edges.restype = i32
     _lib = lib
     return lib
 
@@ -143,6 +148,34 @@ class InteractionNetwork:
         if rc != GNN_OK:
             raise GnnError(rc, "gnn_track_labels")
         return labels
+
+    def load_filter(self, blob: bytes):
+        """Load the filtering MLP (blob of synthetic.pack_filter_blob)."""
+        buf = ctypes.create_string_buffer(blob, len(blob))
+        rc = self.lib.gnn_filter_load(self.handle, buf, len(blob))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_filter_load")
+
+    def filter_edges(self, x, edge_index, threshold: float = 0.5, stream=None):
+        """Filtering step: (scores [E], kept edge index [2, n_kept], kept input ids [n_kept]),
+        all cuda tensors; scores are the filter's, for every input edge."""
+        import torch
+        assert x.is_cuda and x.dtype == torch.float32 and x.is_contiguous()
+        assert edge_index.is_cuda and edge_index.dtype == torch.int32 and edge_index.is_contiguous()
+        E = edge_index.shape[1]
+        scores = torch.empty(E, dtype=torch.float32, device=x.device)
+        kept = torch.empty(2 * max(E, 1), dtype=torch.int32, device=x.device)
+        kept_id = torch.empty(max(E, 1), dtype=torch.int32, device=x.device)
+        n_kept = torch.zeros(1, dtype=torch.int32, device=x.device)
+        rc = self.lib.gnn_filter_edges(self.handle, ctypes.c_void_p(x.data_ptr()),
+                                       ctypes.c_void_p(edge_index.data_ptr()), x.shape[0], E, float(threshold),
+                                       ctypes.c_void_p(scores.data_ptr()), ctypes.c_void_p(kept.data_ptr()),
+                                       ctypes.c_void_p(kept_id.data_ptr()), ctypes.c_void_p(n_kept.data_ptr()),
+                                       _stream_handle(stream))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_filter_edges")
+        n = int(n_kept.item())
+        return scores, kept[:2 * n].view(2, n), kept_id[:n]
 
     def profile(self, on: bool = True):
         self.lib.gnn_profile_enable(self.handle, 1 if on else 0)

@@ -24,6 +24,7 @@
 #include <vector>
 
 #include "../../include/gnn.h"
+#include "compact.cuh"
 #include "components.cuh"
 #include "csr.cuh"
 #include "mlp_tiles.cuh"
@@ -33,6 +34,7 @@ using namespace gnn;
 namespace {
 
 constexpr uint32_t kBlobMagic = 0x57474E47u;
+constexpr uint32_t kFilterMagic = 0x4C464E47u;   // "GNFL": the filtering MLP's weight blob
 constexpr int kHeaderBytes = 8 * 4 + 4 + 4 + 8;
 
 struct Layer { const float* W; const float* b; const float* g; const float* be; int in; };
@@ -45,6 +47,7 @@ struct KernelPlan {          // job list and parameter vectors of one tile-kerne
   int job_acc[kMaxJobs] = {0};
   std::vector<float> vecs;
   float* d_vecs = nullptr;
+  const uint8_t* wmats = nullptr;   // its weight matrices (null: the context's)
 };
 
 }  // namespace
@@ -58,6 +61,11 @@ struct gnn_ctx {
   // plans: 0 node enc -> edge net, 1 node enc -> classifier, 2 edge enc,
   //        3 edge update, 4 node update -> edge net, 5 node update -> classifier, 6 classifier
   KernelPlan plan[7];
+  // filtering step (gnn_filter_load): plan, packed deep-layer matrices, layers, LayerNorm eps
+  KernelPlan filter_plan;
+  uint8_t* d_filter_mats = nullptr;
+  int filter_layers = 0;
+  float filter_eps = 0.f;
   uint32_t* d_err = nullptr;
   // workspace
   void* ws = nullptr;
@@ -126,6 +134,38 @@ void pack_block(const float* W, int ld, int col0, int H, bool with_lo, uint8_t* 
 
 void push(std::vector<float>& v, const float* p, size_t n) { v.insert(v.end(), p, p + n); }
 
+// W' = (I - 11^T/H) W and b' = b - mean(b): the LayerNorm after the layer then sees a
+// zero-mean pre-activation (the fp32 model's kernels compute only the variance).
+void centre_layer(const float* W, const float* b, int H, int in, std::vector<float>& Wc, std::vector<float>& bc) {
+  Wc.resize((size_t)H * in);
+  bc.resize(H);
+  for (int k = 0; k < in; ++k) {
+    double mu = 0.0;
+    for (int n = 0; n < H; ++n) mu += W[(size_t)n * in + k];
+    mu /= H;
+    for (int n = 0; n < H; ++n) Wc[(size_t)n * in + k] = (float)(W[(size_t)n * in + k] - mu);
+  }
+  double mb = 0.0;
+  for (int n = 0; n < H; ++n) mb += b[n];
+  mb /= H;
+  for (int n = 0; n < H; ++n) bc[n] = (float)(b[n] - mb);
+}
+
+// Every whole H-float segment of a plan's vector block is one per-column vector (bias, gamma,
+// beta, head weights, a first-layer weight row); the kernels read them in block-pair order:
+// column 8b + 2q + e at 16*(b/2) + 4q + 2*(b%2) + e.  A trailing partial segment (the head
+// bias) stays as is.  Then padded to 16 bytes.
+void finish_vecs(std::vector<float>& v, int H) {
+  std::vector<float> seg(H);
+  for (size_t base = 0; base + H <= v.size(); base += H) {
+    for (int q = 0; q < 4; ++q)
+      for (int b = 0; b < H / 8; ++b)
+        for (int e = 0; e < 2; ++e) seg[16 * (b / 2) + 4 * q + 2 * (b % 2) + e] = v[base + 8 * b + 2 * q + e];
+    std::copy(seg.begin(), seg.end(), v.begin() + base);
+  }
+  v.resize(padded_vec_floats((int)v.size()), 0.f);
+}
+
 // Test hook: the next g_fail_allocs device allocations made by the library fail (host-side fault
 // injection for the allocation-failure paths; see gnn_debug_fail_allocs).
 std::atomic<int> g_fail_allocs{0};
@@ -157,7 +197,7 @@ int cuda_fail(cudaError_t e) {
   return e == cudaErrorMemoryAllocation ? GNN_ERR_OOM : GNN_ERR_CUDA;
 }
 
-constexpr int kProfGroups = 8;
+constexpr int kProfGroups = 9;
 
 // Returns the record index, or -1 when profiling is off.
 int prof_begin(gnn_ctx* c, int group, int launches, cudaStream_t st) {
@@ -190,6 +230,7 @@ cudaError_t set_all_attrs() {
   if ((e = set_smem_attr<TileKind::EdgeEncoder, H, BF>()) != cudaSuccess) return e;
   if ((e = set_smem_attr<TileKind::EdgeUpdate, H, BF>()) != cudaSuccess) return e;
   if ((e = set_smem_attr<TileKind::NodeUpdate, H, BF>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::Filter, H, BF>()) != cudaSuccess) return e;
   return set_smem_attr<TileKind::Classifier, H, BF>();
 }
 
@@ -199,7 +240,7 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
   for (int j = 0; j < kMaxJobs; ++j) { p.job_mat[j] = pl.job_mat[j]; p.job_acc[j] = pl.job_acc[j]; }
   p.vecs = pl.d_vecs;
   p.n_vec_floats = (int)pl.vecs.size();
-  p.wmats = c->d_mats;
+  p.wmats = pl.wmats ? pl.wmats : c->d_mats;
   p.mat_bytes = c->mat_bytes;
   p.n_tiles = (p.n_rows + kTileRows - 1) / kTileRows;
   if (p.n_tiles == 0) return;
@@ -210,7 +251,7 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
 #ifdef GNN_TRACE
   p.trace = ((int)K == c->trace_kind) ? c->trace : nullptr;
 #endif
-  static const int group[5] = {1, 2, 3, 4, 5};      // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier
+  static const int group[6] = {1, 2, 3, 4, 5, 8};   // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier, Filter
   const int pr = prof_begin(c, group[(int)K], 1, st);
   mlp_tile_kernel<K, H, BF><<<grid, kThreads, smem, st>>>(p);
   prof_end(c, pr, st);
@@ -395,17 +436,8 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
   for (int m = 0; m < N_MLP && !bf; ++m)
     for (int l = 0; l < L; ++l) {
       Layer& ly = lay[m][l];
-      std::vector<float> Wc((size_t)H * ly.in), bc(H);
-      for (int k = 0; k < ly.in; ++k) {
-        double mu = 0.0;
-        for (int n = 0; n < H; ++n) mu += ly.W[(size_t)n * ly.in + k];
-        mu /= H;
-        for (int n = 0; n < H; ++n) Wc[(size_t)n * ly.in + k] = (float)(ly.W[(size_t)n * ly.in + k] - mu);
-      }
-      double mb = 0.0;
-      for (int n = 0; n < H; ++n) mb += ly.b[n];
-      mb /= H;
-      for (int n = 0; n < H; ++n) bc[n] = (float)(ly.b[n] - mb);
+      std::vector<float> Wc, bc;
+      centre_layer(ly.W, ly.b, H, ly.in, Wc, bc);
       centred.push_back(std::move(Wc));
       ly.W = centred.back().data();
       centred.push_back(std::move(bc));
@@ -496,21 +528,7 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
     push(pl.vecs, head_b, 1);
   }
 
-  // Every whole H-float segment of a plan's vector block is one per-column vector (bias, gamma,
-  // beta, head weights, a first-layer weight row); the kernels read them in block-pair order:
-  // column 8b + 2q + e at 16*(b/2) + 4q + 2*(b%2) + e.  A trailing partial segment (the head
-  // bias) stays as is.
-  for (int i = 0; i < 7; ++i) {
-    std::vector<float>& v = c->plan[i].vecs;
-    std::vector<float> seg(H);
-    for (size_t base = 0; base + H <= v.size(); base += H) {
-      for (int q = 0; q < 4; ++q)
-        for (int b = 0; b < H / 8; ++b)
-          for (int e = 0; e < 2; ++e) seg[16 * (b / 2) + 4 * q + 2 * (b % 2) + e] = v[base + 8 * b + 2 * q + e];
-      std::copy(seg.begin(), seg.end(), v.begin() + base);
-    }
-    v.resize(padded_vec_floats((int)v.size()), 0.f);
-  }
+  for (int i = 0; i < 7; ++i) finish_vecs(c->plan[i].vecs, H);
   err = dev_alloc((void**)&c->d_mats, packed.size());
   if (err == cudaSuccess) err = cudaMemcpy(c->d_mats, packed.data(), packed.size(), cudaMemcpyHostToDevice);
   for (int i = 0; i < 7 && err == cudaSuccess; ++i) {
@@ -593,6 +611,112 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
   return gnn_status(ctx, stream);
 }
 
+int gnn_filter_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes) {
+  if (!ctx || !weights_host) return GNN_ERR_INVALID_ARG;
+  const int H = ctx->cfg.hidden, Fn = ctx->cfg.n_node_feat;
+  const bool bf = ctx->cfg.precision == GNN_PRECISION_BF16;
+  if (weights_bytes < (size_t)kHeaderBytes) return GNN_ERR_BAD_WEIGHTS;
+  const uint8_t* blob = (const uint8_t*)weights_host;
+  int32_t hdr[8];
+  float eps;
+  int64_t n_floats;
+  std::memcpy(hdr, blob, 32);
+  std::memcpy(&eps, blob + 32, 4);
+  std::memcpy(&n_floats, blob + 40, 8);
+  const int L = hdr[4];
+  if ((uint32_t)hdr[0] != kFilterMagic || hdr[1] != 1 || hdr[2] != Fn || hdr[3] != H || L < 2 || L > 4 ||
+      hdr[5] != ctx->cfg.precision || !(eps > 0.f))
+    return GNN_ERR_BAD_WEIGHTS;
+  const int64_t want = (int64_t)H * 2 * Fn + 3 * H + (int64_t)(L - 1) * (H * H + 3 * H) + H + 1;
+  if (n_floats != want || weights_bytes != (size_t)kHeaderBytes + 4 * (size_t)want) return GNN_ERR_BAD_WEIGHTS;
+  const float* f = (const float*)(blob + kHeaderBytes);
+  std::vector<Layer> lay(L);
+  for (int l = 0; l < L; ++l) {
+    const int in = l == 0 ? 2 * Fn : H;
+    lay[l] = {f, f + (size_t)H * in, f + (size_t)H * in + H, f + (size_t)H * in + 2 * H, in};
+    f += (size_t)H * in + 3 * H;
+  }
+  const float* head = f;
+  std::vector<std::vector<float>> centred(2 * L);
+  if (!bf)
+    for (int l = 0; l < L; ++l) {
+      centre_layer(lay[l].W, lay[l].b, H, lay[l].in, centred[2 * l], centred[2 * l + 1]);
+      lay[l].W = centred[2 * l].data();
+      lay[l].b = centred[2 * l + 1].data();
+    }
+  KernelPlan pl;
+  for (int l = 1; l < L; ++l) { pl.job_acc[pl.n_jobs] = 0; pl.job_mat[pl.n_jobs] = l - 1; ++pl.n_jobs; }
+  for (int k = 0; k < 2 * Fn; ++k)                   // first-layer weight, transposed
+    for (int i = 0; i < H; ++i) pl.vecs.push_back(lay[0].W[(size_t)i * 2 * Fn + k]);
+  for (int l = 0; l < L; ++l) { push(pl.vecs, lay[l].b, H); push(pl.vecs, lay[l].g, H); push(pl.vecs, lay[l].be, H); }
+  push(pl.vecs, head, H + 1);
+  finish_vecs(pl.vecs, H);
+  std::vector<uint8_t> packed((size_t)ctx->mat_bytes * (L - 1));
+  for (int l = 1; l < L; ++l) pack_block(lay[l].W, H, 0, H, !bf, packed.data() + (size_t)(l - 1) * ctx->mat_bytes);
+  // replace a previous filter
+  if (ctx->filter_plan.d_vecs) { cudaFree(ctx->filter_plan.d_vecs); ctx->filter_plan.d_vecs = nullptr; }
+  if (ctx->d_filter_mats) { cudaFree(ctx->d_filter_mats); ctx->d_filter_mats = nullptr; }
+  ctx->filter_layers = 0;
+  cudaError_t err = dev_alloc((void**)&ctx->d_filter_mats, packed.size());
+  if (err == cudaSuccess) err = cudaMemcpy(ctx->d_filter_mats, packed.data(), packed.size(), cudaMemcpyHostToDevice);
+  if (err == cudaSuccess) err = dev_alloc((void**)&pl.d_vecs, pl.vecs.size() * 4);
+  if (err == cudaSuccess) err = cudaMemcpy(pl.d_vecs, pl.vecs.data(), pl.vecs.size() * 4, cudaMemcpyHostToDevice);
+  if (err != cudaSuccess) {
+    if (pl.d_vecs) cudaFree(pl.d_vecs);
+    if (ctx->d_filter_mats) { cudaFree(ctx->d_filter_mats); ctx->d_filter_mats = nullptr; }
+    return cuda_fail(err);
+  }
+  pl.wmats = ctx->d_filter_mats;
+  ctx->filter_plan = std::move(pl);
+  ctx->filter_layers = L;
+  ctx->filter_eps = eps;
+  return GNN_OK;
+}
+
+int gnn_filter_edges(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
+                     int64_t n_edges, float threshold, float* edge_scores, int32_t* kept_index, int32_t* kept_id,
+                     int32_t* n_kept, gnn_stream_t stream) {
+  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX || !n_kept)
+    return GNN_ERR_INVALID_ARG;
+  if (ctx->filter_layers == 0) return GNN_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (n_edges == 0) {
+    const cudaError_t err = cudaMemsetAsync(n_kept, 0, sizeof(int32_t), st);
+    return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+  }
+  if (n_nodes == 0 || !node_feats || !edge_index || !edge_scores || !kept_index) return GNN_ERR_INVALID_ARG;
+  int rc = ensure_workspace(ctx, n_nodes, n_edges);          // block counts live in the sort keys' buffer
+  if (rc != GNN_OK) return rc;
+  const int N = (int)n_nodes, E = (int)n_edges;
+  TileParams p{};
+  p.n_rows = E;
+  p.n_nodes = N;
+  p.n_layers = ctx->filter_layers;
+  p.n_feat = ctx->cfg.n_node_feat;
+  p.eps = ctx->filter_eps;
+  p.x = node_feats;
+  p.x_stride = ctx->cfg.n_node_feat;
+  p.ei_in = edge_index;
+  p.scores = edge_scores;
+  p.err = ctx->d_err;
+  const bool bf = ctx->cfg.precision == GNN_PRECISION_BF16;
+  if (ctx->cfg.hidden == 128) {
+    if (bf) launch_tile<TileKind::Filter, 128, true>(ctx, ctx->filter_plan, p, st);
+    else launch_tile<TileKind::Filter, 128, false>(ctx, ctx->filter_plan, p, st);
+  } else {
+    if (bf) launch_tile<TileKind::Filter, 64, true>(ctx, ctx->filter_plan, p, st);
+    else launch_tile<TileKind::Filter, 64, false>(ctx, ctx->filter_plan, p, st);
+  }
+  const int nb = (E + kCompactBlock - 1) / kCompactBlock;
+  int* counts = ctx->keys_a;
+  compact_count_kernel<<<nb, kCompactThreads, 0, st>>>(edge_scores, E, threshold, counts);
+  compact_scan_kernel<<<1, 1024, 0, st>>>(counts, nb, n_kept);
+  compact_scatter_kernel<<<nb, kCompactThreads, 0, st>>>(edge_scores, edge_index, E, threshold, counts, n_kept,
+                                                          kept_index, kept_id);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
+
 int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge_index, int64_t n_nodes,
                      int64_t n_edges, float threshold, int32_t* labels, gnn_stream_t stream) {
   if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX) return GNN_ERR_INVALID_ARG;
@@ -673,6 +797,8 @@ void gnn_destroy(gnn_ctx* ctx) {
   if (ctx->d_mats) cudaFree(ctx->d_mats);
   for (int i = 0; i < 7; ++i)
     if (ctx->plan[i].d_vecs) cudaFree(ctx->plan[i].d_vecs);
+  if (ctx->filter_plan.d_vecs) cudaFree(ctx->filter_plan.d_vecs);
+  if (ctx->d_filter_mats) cudaFree(ctx->d_filter_mats);
   if (ctx->d_err) cudaFree(ctx->d_err);
   if (ctx->stage) cudaFree(ctx->stage);
   for (auto& r : ctx->prof) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }

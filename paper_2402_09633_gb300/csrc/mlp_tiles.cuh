@@ -44,6 +44,7 @@ enum class TileKind : int {
   EdgeUpdate  = 2,     // e <- MLP_edge([h_src, h_dst, e]) via e*W_e + P_s[src] + P_d[dst]
   NodeUpdate  = 3,     // h <- MLP_node([h, sum of incoming e]); then P_s, P_d of new h
   Classifier  = 4,     // score = sigmoid(w_o . MLP_cls([h_src, h_dst, e]) + b_o)
+  Filter      = 5,     // filtering step: score = sigmoid(w_o . MLP_f([x_src, x_dst]) + b_o), input edge order
 };
 
 constexpr int kThreads = 640;
@@ -87,6 +88,7 @@ struct TileParams {
   void* agg;                  // [N, H] row-tiled: sum of incoming messages per node; fp32 or bf16
   float* scores;              // [E] input order
   uint32_t* err;              // device error word
+  const int32_t* ei_in;       // filter: [2, E] input edge index (rows in input order)
 #ifdef GNN_TRACE
   unsigned long long* trace;  // [3 roles][kTraceEvents] %globaltimer stamps of CTA 0
 #endif
@@ -713,6 +715,69 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           const float* vl = vb + 3 * (L - 1) * H;
           const bool w0 = ok && ok0, w1 = ok && ok1;
           ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { store_t16_chunk(p.e, row0, w0, w1, k, t); });
+        }
+      } else if constexpr (KIND == TileKind::Filter) {
+        // vec layout: [W1^T (2 F_n x H), b1, gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]
+        // Layer 1 on CUDA cores from the raw features of both endpoints, [x_src, x_dst].
+        bool valid[2] = {false, false};
+        int sv[2] = {0, 0}, dv[2] = {0, 0};
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int row = r ? row1 : row0;
+          if (r ? ok1 : ok0) {
+            const int s = p.ei_in[row], d = p.ei_in[(size_t)p.n_rows + row];
+            valid[r] = s >= 0 && s < p.n_nodes && d >= 0 && d < p.n_nodes;
+            sv[r] = valid[r] ? s : 0;
+            dv[r] = valid[r] ? d : 0;
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < 4 * NB; ++i) v[i] = 0.f;
+        for (int k = 0; k < 2 * p.n_feat; ++k) {
+          const int node0 = k < p.n_feat ? sv[0] : dv[0], node1 = k < p.n_feat ? sv[1] : dv[1];
+          const int col = k < p.n_feat ? k : k - p.n_feat;
+          const float x0 = valid[0] ? p.x[(size_t)node0 * p.x_stride + col] : 0.f;
+          const float x1 = valid[1] ? p.x[(size_t)node1 * p.x_stride + col] : 0.f;
+#pragma unroll
+          for (int b = 0; b < NB; b += 2) {
+            const float4 w = vq4(vecs + k * H, b);
+            v[4 * b] = fmaf(w.x, x0, v[4 * b]); v[4 * b + 1] = fmaf(w.y, x0, v[4 * b + 1]);
+            v[4 * b + 2] = fmaf(w.x, x1, v[4 * b + 2]); v[4 * b + 3] = fmaf(w.y, x1, v[4 * b + 3]);
+            v[4 * b + 4] = fmaf(w.z, x0, v[4 * b + 4]); v[4 * b + 5] = fmaf(w.w, x0, v[4 * b + 5]);
+            v[4 * b + 6] = fmaf(w.z, x1, v[4 * b + 6]); v[4 * b + 7] = fmaf(w.w, x1, v[4 * b + 7]);
+          }
+        }
+        const float* vb = vecs + 2 * p.n_feat * H;
+        add_vec(v, vb);
+        ln_relu(v, vb + H, vb + 2 * H);
+        for (int l = 2; l <= L; ++l) {
+          put_a(v);
+          arrive_a(j, seq); next_job();
+          wait_job();
+          load_d(v);
+          const float* vl = vb + 3 * (l - 1) * H;
+          add_vec(v, vl);
+          ln_relu(v, vl + H, vl + 2 * H);
+        }
+        const float* wo = vb + 3 * L * H;
+        if constexpr (BF) {                  // the head's input is a bf16 activation
+#pragma unroll
+          for (int i = 0; i < 4 * NB; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+        }
+        float z0 = 0.f, z1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < NB; k += 2) {
+          const float4 w = vq4(wo, k);
+          z0 = fmaf(v[4 * k], w.x, fmaf(v[4 * k + 1], w.y, fmaf(v[4 * k + 4], w.z, fmaf(v[4 * k + 5], w.w, z0))));
+          z1 = fmaf(v[4 * k + 2], w.x, fmaf(v[4 * k + 3], w.y, fmaf(v[4 * k + 6], w.z, fmaf(v[4 * k + 7], w.w, z1))));
+        }
+        z0 = quad_sum(z0) + wo[H];
+        z1 = quad_sum(z1) + wo[H];
+        if (ok && (lane & 3) == 0) {
+          const float nan = __int_as_float(0x7fc00000);
+          if (ok0) p.scores[row0] = valid[0] ? 1.0f / (1.0f + __expf(-z0)) : nan;
+          if (ok1) p.scores[row1] = valid[1] ? 1.0f / (1.0f + __expf(-z1)) : nan;
+          if ((ok0 && !valid[0]) || (ok1 && !valid[1])) atomicOr(p.err, DEV_ERR_INDEX_RANGE);
         }
       } else {
         // NodeEncoder / NodeUpdate.

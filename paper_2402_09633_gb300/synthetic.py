@@ -292,3 +292,45 @@ def blob_n_floats(cfg: ModelConfig) -> int:
     for name, fan_in in cfg.mlp_in_dims().items():
         n += H * fan_in + 3 * H + (L - 1) * (H * H + 3 * H)
     return n + H + 1
+
+
+# --------------------------------------------------------------------------- filtering MLP
+
+FILTER_MAGIC = 0x4C464E47  # "GNFL" little-endian
+
+
+def init_filter_weights(cfg: ModelConfig, seed: int = 1) -> dict:
+    """Random-init filtering MLP on [x_src, x_dst] (2 * n_node_feat inputs): layers of the same
+    kind and draws as init_weights, then head w_o ~ N(0, 1/H), b_o = 0; rounded to bf16 for the
+    bf16 model."""
+    rng = np.random.default_rng(seed)
+    H = cfg.hidden
+    fan_in = 2 * cfg.n_node_feat
+    layers = []
+    for _ in range(cfg.mlp_layers):
+        W = (rng.standard_normal((H, fan_in)) / np.sqrt(fan_in)).astype(np.float32)
+        b = (0.1 * rng.standard_normal(H)).astype(np.float32)
+        g = (1.0 + 0.1 * rng.standard_normal(H)).astype(np.float32)
+        be = (0.1 * rng.standard_normal(H)).astype(np.float32)
+        layers.append((W, b, g, be))
+        fan_in = H
+    out = {"layers": layers, "head_w": (rng.standard_normal(H) / np.sqrt(H)).astype(np.float32),
+           "head_b": np.zeros(1, np.float32)}
+    if cfg.precision == PRECISION_BF16:
+        out = {"layers": [tuple(_round_bf16(t) for t in lay) for lay in layers],
+               "head_w": _round_bf16(out["head_w"]), "head_b": _round_bf16(out["head_b"])}
+    return out
+
+
+def pack_filter_blob(cfg: ModelConfig, fw: dict) -> bytes:
+    """Filter blob: 8 int32 (magic, version 1, n_node_feat, hidden, mlp_layers, precision, 0, 0),
+    float32 ln_eps, int32 0, int64 float count; per layer W [H, in], b, gamma, beta; w_o, b_o."""
+    arrays = []
+    for (W, b, g, be) in fw["layers"]:
+        arrays += [W, b, g, be]
+    arrays += [fw["head_w"], fw["head_b"]]
+    payload = b"".join(np.ascontiguousarray(a, dtype="<f4").tobytes() for a in arrays)
+    header = struct.pack("<8i f i q", FILTER_MAGIC, 1, cfg.n_node_feat, cfg.hidden, len(fw["layers"]),
+                         cfg.precision, 0, 0, cfg.ln_eps, 0, len(payload) // 4)
+    return header + payload
+

@@ -426,3 +426,32 @@ def test_track_labels_against_library_components():
     smallest = np.full(comp.max() + 1, n)
     np.minimum.at(smallest, comp, np.arange(n))
     np.testing.assert_array_equal(O.track_labels(sc, ei, n, 0.3), smallest[comp])
+
+
+# ------------------------------------------------------------- filtering
+
+def test_filter_scores_by_hand():
+    """One layer, H = 2, F_n = 1: s = sigmoid(w . ReLU(LN(W [x_src, x_dst] + b)) + b_o)."""
+    fw = {"layers": [(np.array([[1.0, -2.0], [0.5, 1.5]]), np.array([0.1, -0.3]), np.array([2.0, 0.5]),
+                      np.array([-0.1, 0.05]))],
+          "head_w": np.array([1.5, -0.75]), "head_b": np.array([0.2])}
+    x = np.array([[0.4], [-0.3], [0.9]], np.float32)
+    ei = np.array([[0, 2, 1, 0], [1, 0, 2, 5]], np.int32)            # the last edge is out of range
+    got_s, got_z = O.filter_scores(fw, x, ei, HAND_EPS, return_logits=True)
+    for k in range(3):
+        a, b = float(x[ei[0, k], 0]), float(x[ei[1, k], 0])
+        v1, v2 = a - 2.0 * b + 0.1, 0.5 * a + 1.5 * b - 0.3
+        h = _relu2(_ln2(v1, v2, (2.0, 0.5), (-0.1, 0.05)))
+        z = 1.5 * h[0] - 0.75 * h[1] + 0.2
+        assert abs(got_z[k] - z) < 1e-12 and abs(got_s[k] - 1.0 / (1.0 + math.exp(-z))) < 1e-12
+    assert np.isnan(got_s[3]) and np.isnan(got_z[3])
+    # swapping source and destination changes the score (the input is ordered [x_src, x_dst])
+    assert abs(O.filter_scores(fw, x, ei[::-1, :1], HAND_EPS)[0] - got_s[0]) > 1e-3
+
+
+def test_apply_filtering_keeps_order_and_drops_nan():
+    ei = np.array([[0, 1, 2, 3, 4], [5, 6, 7, 8, 9]], np.int32)
+    sc = np.array([0.9, 0.2, np.nan, 0.51, 0.5])
+    kept, ids = O.apply_filtering(sc, ei, 0.5)
+    assert ids.tolist() == [0, 3]
+    assert kept.tolist() == [[0, 3], [5, 8]]
