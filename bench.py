@@ -72,12 +72,13 @@ def step_model(w: S.Workload):
 # ------------------------------------------------------------------ ncu traffic
 PROFILE_FOR_KERNEL = {("edge_update", False): "edge_update_full_event.md",
                       ("edge_update", True): "edge_update_bf16_full_event.md"}
-KERNEL_SOURCES = ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh", "gnn_api.cu")
+KERNEL_SOURCES = ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh")
 
 
 def source_hash() -> str:
-    """First 16 hex digits of a sha256 over the kernel sources' code: `//` comments, trailing
-    blanks and empty lines are left out, so editing a comment does not void a profile."""
+    """First 16 hex digits of a sha256 over the code of the sources that define the profiled
+    kernels and their launch geometry (the host API around them is left out): `//` comments,
+    trailing blanks and empty lines are skipped, so editing a comment does not void a profile."""
     import hashlib
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:

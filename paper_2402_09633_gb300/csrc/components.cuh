@@ -54,6 +54,14 @@ __global__ void cc_union_kernel(const float* __restrict__ scores, const int32_t*
   }
 }
 
+// Shortens the forest before the final pass: every node points at the root its (path-halving)
+// walk reached.  Racing halving stores can leave some nodes one or more steps below their root,
+// so this pass alone does not give the labels; it only makes the read-only walks short.
+__global__ void cc_compress_kernel(int32_t* parent, int n) {
+  const int v = blockIdx.x * blockDim.x + threadIdx.x;
+  if (v < n) parent[v] = cc_find(parent, v);
+}
+
 // labels[v] = root of v (the smallest id of its component).  The walk only reads: a path-halving
 // store from another thread could otherwise land on parent[v] after v has written its root and
 // leave v pointing at an intermediate ancestor.  Every value a reader meets is an ancestor (an

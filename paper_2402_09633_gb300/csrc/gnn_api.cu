@@ -244,10 +244,8 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
   p.mat_bytes = c->mat_bytes;
   p.n_tiles = (p.n_rows + kTileRows - 1) / kTileRows;
   if (p.n_tiles == 0) return;
-  uint32_t smem = tile_smem_bytes<H, BF>(p.n_vec_floats);
-  if (smem < 120 * 1024) smem = 120 * 1024;           // one CTA per SM (it owns the TMEM)
-  const int pairs = (p.n_tiles + 1) / 2;
-  const int grid = pairs < c->n_sm ? pairs : c->n_sm;
+  const uint32_t smem = tile_launch_smem<H, BF>(p.n_vec_floats);
+  const int grid = tile_grid(p.n_tiles, c->n_sm);
 #ifdef GNN_TRACE
   p.trace = ((int)K == c->trace_kind) ? c->trace : nullptr;
 #endif
@@ -726,6 +724,7 @@ int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge
   const int N = (int)n_nodes, E = (int)n_edges, tb = 256;
   cc_init_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
   if (E > 0) cc_union_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(edge_scores, edge_index, N, E, threshold, labels, ctx->d_err);
+  cc_compress_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
   cc_flatten_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);

@@ -131,6 +131,17 @@ constexpr uint32_t tile_smem_bytes(int n_vec_floats) {
   return TileGeom<H, BF>::RING_BYTES + (uint32_t)padded_vec_floats(n_vec_floats) * 4u + 256 + 1024;
 }
 
+// Launch geometry: dynamic shared memory of at least 120 KB, so that one CTA per SM runs (it owns
+// the TMEM), and one persistent CTA per SM or per tile pair, whichever is fewer.
+template <int H, bool BF>
+constexpr uint32_t tile_launch_smem(int n_vec_floats) {
+  return tile_smem_bytes<H, BF>(n_vec_floats) < 120u * 1024u ? 120u * 1024u : tile_smem_bytes<H, BF>(n_vec_floats);
+}
+inline int tile_grid(int n_tiles, int n_sm) {
+  const int pairs = (n_tiles + 1) / 2;
+  return pairs < n_sm ? pairs : n_sm;
+}
+
 // ----------------------------------------------------------------- kernel
 template <TileKind KIND, int H, bool BF>
 __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams p) {
