@@ -48,6 +48,7 @@ enum gnn_status_code {
   GNN_ERR_CUDA = -4,           /* a CUDA runtime call or kernel launch failed */
   GNN_ERR_INDEX_RANGE = -5,    /* device: an edge endpoint was outside [0, n_nodes) */
   GNN_ERR_DEVICE_TIMEOUT = -6, /* device: a pipeline wait expired; results are invalid */
+  GNN_ERR_CAPACITY = -7,       /* device: an output buffer was too small (gnn_build_graph) */
 };
 
 enum gnn_precision {
@@ -132,6 +133,44 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
                    int64_t n_edges, float* edge_scores, gnn_stream_t stream);
 
 /*
+ * gnn_embed_load -- load the embedding MLP (paper Section 2.1: the first step maps every space
+ * point's raw features into a latent space where hits of one track lie close together).  Network:
+ * y = normalize(W_out . MLP_L(x) + b_out), L hidden layers Linear -> LayerNorm -> ReLU of the
+ * context's hidden width, then a Linear to D outputs, scaled to unit length (a zero vector stays
+ * zero).  Blob (little-endian, copied): eight int32 (magic 0x4D454E47 "GNEM", version 1,
+ * n_node_feat, hidden, L (2..4), precision, D (1..16), reserved), float32 ln_eps, int32 reserved,
+ * int64 float count, then per hidden layer W [H, in] row-major, b, gamma, beta (in = n_node_feat
+ * for layer 1, H afterwards), then W_out [D, H], b_out [D].  n_node_feat, hidden and precision
+ * must equal the context's.  A later call replaces it.  Errors: INVALID_ARG, BAD_WEIGHTS, OOM, CUDA.
+ *
+ * gnn_embed -- embedding of every hit: node_feats device float32 [n_nodes, n_node_feat] in,
+ * embedding device float32 [n_nodes, D] out (caller-owned).  Enqueued on `stream`.  Errors:
+ * INVALID_ARG (no embedding loaded, null pointer, bad size), CUDA.
+ *
+ * gnn_build_graph -- candidate edges by fixed-radius neighbours in the embedding space (Section
+ * 2.1: the graph is built between hits closer than a radius in the latent space).  Every pair of
+ * hits whose squared distance, summed over the emb_dim coordinates in order in fp32 with one
+ * rounding per product and per sum, is below radius * radius (rounded to fp32) becomes one edge,
+ * oriented from the hit with the smaller r (node_feats column 0; the smaller id on a tie).
+ *   embedding  device float32 [n_nodes, emb_dim], emb_dim 1..16; unit vectors (as gnn_embed
+ *              writes them) are searched on a grid over [-1, 1]^3, other values stay exact but
+ *              crowd into the grid's edge cells
+ *   node_feats device float32 [n_nodes, n_node_feat] (column 0 orients the edges)
+ *   edge_index device int32 with room for [2, max_edges], output: contiguous [2, n_edges]
+ *   n_edges    device int32 [1], output: the number of edges found
+ * When n_edges exceeds max_edges nothing is written to edge_index, *n_edges still holds the
+ * count (saturated at INT32_MAX), and gnn_status reports GNN_ERR_CAPACITY: call again with room
+ * for that many.  The order
+ * of the edges is deterministic.  Uses a scratch buffer of the context (grown on demand,
+ * synchronous then).  Errors: INVALID_ARG (radius <= 0, emb_dim out of range, null pointer, bad
+ * sizes), OOM, CUDA.
+ */
+int gnn_embed_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes);
+int gnn_embed(gnn_ctx* ctx, const float* node_feats, int64_t n_nodes, float* embedding, gnn_stream_t stream);
+int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const float* node_feats, int64_t n_nodes,
+                    float radius, int64_t max_edges, int32_t* edge_index, int32_t* n_edges, gnn_stream_t stream);
+
+/*
  * gnn_filter_load -- load the filtering MLP (paper Section 2.1: the step before the GNN scores every
  * candidate edge from the raw features of its two hits; applyFiltering then drops the edges below
  * a fixed threshold).  Network: s = sigmoid(w_o . MLP_L([x_src, x_dst]) + b_o), each of its L
@@ -193,8 +232,8 @@ int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge
  * kernel launches launches[g]; then clear the records.  Groups: 0 CSR build
  * (all its kernels), 1 node encoder, 2 edge encoder, 3 edge update, 4 node
  * update, 5 classifier, 6 host<->device copies of gnn_infer_host, 7 message
- * aggregation, 8 filtering MLP.  Either output pointer may be NULL.  Returns
- * the number of groups (9) or an error.
+ * aggregation, 8 filtering MLP, 9 embedding MLP.  Either output pointer may
+ * be NULL.  Returns the number of groups (10) or an error.
  */
 int gnn_profile_enable(gnn_ctx* ctx, int on);
 int gnn_profile_read(gnn_ctx* ctx, double* ms, int64_t* launches, int n_groups);

@@ -211,3 +211,45 @@ def apply_filtering(scores: np.ndarray, edge_index: np.ndarray, threshold: float
     ids = np.nonzero(keep)[0]
     return np.asarray(edge_index)[:, ids], ids
 
+
+def embed(ew: dict, x: np.ndarray, eps: float = 1e-5, bf16: bool = False) -> np.ndarray:
+    """Embedding step (Section 2.1: an MLP maps every space point's raw features into a latent
+    space): y = normalize(W_out . MLP(x) + b_out), unit length (a zero vector stays zero)."""
+    v = mlp(np.asarray(x, np.float64), ew["layers"], eps, round_bf16 if bf16 else None)
+    z = v @ np.asarray(ew["out_w"], np.float64).T + np.asarray(ew["out_b"], np.float64)
+    n = np.sqrt((z * z).sum(axis=1, keepdims=True))
+    return np.where(n > 0, z / np.where(n > 0, n, 1.0), 0.0)
+
+
+def sq_dist_f32(a: np.ndarray, b: np.ndarray) -> np.ndarray:
+    """Squared distances of float32 row pairs, summed over the coordinates in order with one
+    float32 rounding per product and per sum."""
+    a = np.asarray(a, np.float32)
+    b = np.asarray(b, np.float32)
+    s = np.zeros(a.shape[0], np.float32)
+    for d in range(a.shape[1]):
+        diff = (a[:, d] - b[:, d]).astype(np.float32)
+        s = (s + (diff * diff).astype(np.float32)).astype(np.float32)
+    return s
+
+
+def radius_graph(emb: np.ndarray, r_col: np.ndarray, radius: float, candidates=None) -> np.ndarray:
+    """Graph building (Section 2.1: edges between hits closer than a radius in the latent space):
+    every pair {i, j} whose float32 squared distance (sq_dist_f32) is below float32(radius)^2
+    (rounded to float32), oriented from the smaller r (r_col; the smaller index on a tie) to the
+    other.  Returns the edges as an [n, 2] array sorted by (src, dst).  `candidates` ([m, 2], i < j)
+    may restrict the pairs tested (a superset of the answer); by default every pair is tested."""
+    emb = np.asarray(emb, np.float32)
+    n = emb.shape[0]
+    if candidates is None:
+        ii, jj = np.triu_indices(n, 1)
+    else:
+        ii, jj = candidates[:, 0], candidates[:, 1]
+    r2 = np.float32(np.float32(radius) * np.float32(radius))
+    keep = sq_dist_f32(emb[ii], emb[jj]) < r2
+    i, j = ii[keep], jj[keep]
+    r = np.asarray(r_col, np.float32)
+    first = (r[i] < r[j]) | ((r[i] == r[j]) & (i < j))
+    e = np.stack([np.where(first, i, j), np.where(first, j, i)], axis=1).astype(np.int64)
+    return e[np.lexsort((e[:, 1], e[:, 0]))] if e.size else e.reshape(0, 2)
+

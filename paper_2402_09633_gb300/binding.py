@@ -5,6 +5,7 @@ computation runs in the library's CUDA kernels."""
 from __future__ import annotations
 
 import ctypes
+import struct
 import os
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -13,13 +14,13 @@ _lib = None
 
 GNN_OK = 0
 ERRORS = {-1: "INVALID_ARG", -2: "BAD_WEIGHTS", -3: "OOM", -4: "CUDA", -5: "INDEX_RANGE",
-          -6: "DEVICE_TIMEOUT"}
+          -6: "DEVICE_TIMEOUT", -7: "CAPACITY"}
 EXPORTED = ("gnn_create", "gnn_reserve", "gnn_infer", "gnn_infer_host", "gnn_status",
             "gnn_destroy", "gnn_error_string", "gnn_debug_copy", "gnn_profile_enable",
             "gnn_profile_read", "gnn_track_labels", "gnn_csr_build_noalloc", "gnn_filter_load",
-            "gnn_filter_edges")
+            "gnn_filter_edges", "gnn_embed_load", "gnn_embed", "gnn_build_graph")
 PROFILE_GROUPS = ("csr_build", "node_encoder", "edge_encoder", "edge_update", "node_update",
-                  "classifier", "host_copies", "aggregate", "filter")
+                  "classifier", "host_copies", "aggregate", "filter", "embed")
 
 
 class GnnError(RuntimeError):
@@ -70,6 +71,12 @@ def load_library(path: str = LIB_PATH):
     lib.gnn_filter_load.restype = i32
     lib.gnn_filter_edges.argtypes = [vp, vp, vp, i64, i64, ctypes.c_float, vp, vp, vp, vp, vp]
     lib.gnn_filter_edges.restype = i32
+    lib.gnn_embed_load.argtypes = [vp, vp, ctypes.c_size_t]
+    lib.gnn_embed_load.restype = i32
+    lib.gnn_embed.argtypes = [vp, vp, i64, vp, vp]
+    lib.gnn_embed.restype = i32
+    lib.gnn_build_graph.argtypes = [vp, vp, i32, vp, i64, ctypes.c_float, i64, vp, vp, vp]
+    lib.gnn_build_graph.restype = i32
     _lib = lib
     return lib
 
@@ -148,6 +155,46 @@ class InteractionNetwork:
         if rc != GNN_OK:
             raise GnnError(rc, "gnn_track_labels")
         return labels
+
+    def load_embedding(self, blob: bytes):
+        """Load the embedding MLP (blob of synthetic.pack_embed_blob)."""
+        buf = ctypes.create_string_buffer(blob, len(blob))
+        rc = self.lib.gnn_embed_load(self.handle, buf, len(blob))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_embed_load")
+        self.embed_dim = struct.unpack_from("<8i", blob)[6]
+
+    def embed(self, x, stream=None):
+        """Embedding [N, dim] (cuda float32) of every hit; dim is the loaded embedding MLP's."""
+        import torch
+        assert x.is_cuda and x.dtype == torch.float32 and x.is_contiguous()
+        out = torch.empty((x.shape[0], getattr(self, "embed_dim", 1)), dtype=torch.float32, device=x.device)
+        rc = self.lib.gnn_embed(self.handle, ctypes.c_void_p(x.data_ptr()), x.shape[0],
+                                ctypes.c_void_p(out.data_ptr()), _stream_handle(stream))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_embed")
+        return out
+
+    def build_graph(self, emb, x, radius: float, max_edges: int, stream=None):
+        """Fixed-radius candidate edges: (edge index [2, n] cuda int32, n).  Raises GnnError
+        (CAPACITY) when more than max_edges edges exist, with the number found as .n_edges."""
+        import torch
+        assert emb.is_cuda and emb.dtype == torch.float32 and emb.is_contiguous()
+        out = torch.empty(2 * max(max_edges, 1), dtype=torch.int32, device=emb.device)
+        n = torch.zeros(1, dtype=torch.int32, device=emb.device)
+        rc = self.lib.gnn_build_graph(self.handle, ctypes.c_void_p(emb.data_ptr()), emb.shape[1],
+                                      ctypes.c_void_p(x.data_ptr()), emb.shape[0], float(radius), max_edges,
+                                      ctypes.c_void_p(out.data_ptr()), ctypes.c_void_p(n.data_ptr()),
+                                      _stream_handle(stream))
+        if rc != GNN_OK:
+            raise GnnError(rc, "gnn_build_graph")
+        st = self.status(stream)
+        k = int(n.item())
+        if st != GNN_OK:
+            err = GnnError(st, "gnn_build_graph")
+            err.n_edges = k
+            raise err
+        return out[:2 * k].view(2, k), k
 
     def load_filter(self, blob: bytes):
         """Load the filtering MLP (blob of synthetic.pack_filter_blob)."""

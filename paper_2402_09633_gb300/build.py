@@ -12,7 +12,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libgnn_gb300.so")
 SOURCES = [os.path.join(HERE, "csrc", "gnn_api.cu")]
-DEPS = SOURCES + [os.path.join(HERE, "csrc", f) for f in ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh", "components.cuh")] + \
+DEPS = SOURCES + [os.path.join(HERE, "csrc", f) for f in ("ptx.cuh", "csr.cuh", "mlp_tiles.cuh", "components.cuh", "compact.cuh", "frnn.cuh")] + \
     [os.path.join(ROOT, "include", "gnn.h")]
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc")
 FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-lineinfo", "-std=c++17",

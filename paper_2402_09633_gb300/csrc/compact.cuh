@@ -39,39 +39,42 @@ __global__ void __launch_bounds__(kCompactThreads) compact_count_kernel(const fl
 }
 
 // Exclusive scan of the block counts in place (one block of 1024 threads); the total goes to *total.
+// The sums are taken in 64 bits and the total saturates at INT32_MAX, so a caller that compares the
+// total with its capacity (below INT32_MAX) sees an overflow as "too many" (offsets past the
+// overflow point are then meaningless and must not be used).
 __global__ void __launch_bounds__(1024) compact_scan_kernel(int* __restrict__ counts, int n_blocks,
                                                             int* __restrict__ total) {
-  __shared__ int wsum[32];
-  __shared__ int carry;
+  __shared__ long long wsum[32];
+  __shared__ long long carry;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   if (t == 0) carry = 0;
   __syncthreads();
   for (int base = 0; base < n_blocks; base += 1024) {
     const int i = base + t;
-    const int v = i < n_blocks ? counts[i] : 0;
-    int x = v;                                             // inclusive scan inside the warp
+    const long long v = i < n_blocks ? counts[i] : 0;
+    long long x = v;                                       // inclusive scan inside the warp
     for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      const long long y = __shfl_up_sync(0xffffffffu, x, o);
       if (lane >= o) x += y;
     }
     if (lane == 31) wsum[warp] = x;
     __syncthreads();
     if (warp == 0) {
-      int w = wsum[lane];
+      long long w = wsum[lane];
       for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, w, o);
+        const long long y = __shfl_up_sync(0xffffffffu, w, o);
         if (lane >= o) w += y;
       }
       wsum[lane] = w;                                      // inclusive over warps
     }
     __syncthreads();
-    const int excl = carry + (warp > 0 ? wsum[warp - 1] : 0) + x - v;
-    if (i < n_blocks) counts[i] = excl;
+    const long long excl = carry + (warp > 0 ? wsum[warp - 1] : 0) + x - v;
+    if (i < n_blocks) counts[i] = (int)excl;
     __syncthreads();
     if (t == 0) carry += wsum[31];
     __syncthreads();
   }
-  if (t == 0) *total = carry;
+  if (t == 0) *total = carry > 0x7fffffffLL ? 0x7fffffff : (int)carry;
 }
 
 __global__ void __launch_bounds__(kCompactThreads) compact_scatter_kernel(

@@ -27,6 +27,7 @@
 #include "compact.cuh"
 #include "components.cuh"
 #include "csr.cuh"
+#include "frnn.cuh"
 #include "mlp_tiles.cuh"
 
 using namespace gnn;
@@ -35,6 +36,7 @@ namespace {
 
 constexpr uint32_t kBlobMagic = 0x57474E47u;
 constexpr uint32_t kFilterMagic = 0x4C464E47u;   // "GNFL": the filtering MLP's weight blob
+constexpr uint32_t kEmbedMagic = 0x4D454E47u;    // "GNEM": the embedding MLP's weight blob
 constexpr int kHeaderBytes = 8 * 4 + 4 + 4 + 8;
 
 struct Layer { const float* W; const float* b; const float* g; const float* be; int in; };
@@ -66,6 +68,13 @@ struct gnn_ctx {
   uint8_t* d_filter_mats = nullptr;
   int filter_layers = 0;
   float filter_eps = 0.f;
+  // embedding step (gnn_embed_load) and graph building scratch
+  KernelPlan embed_plan;
+  uint8_t* d_embed_mats = nullptr;
+  int embed_layers = 0, embed_dim = 0;
+  float embed_eps = 0.f;
+  int* aux = nullptr;
+  size_t aux_ints = 0;
   uint32_t* d_err = nullptr;
   // workspace
   void* ws = nullptr;
@@ -197,7 +206,7 @@ int cuda_fail(cudaError_t e) {
   return e == cudaErrorMemoryAllocation ? GNN_ERR_OOM : GNN_ERR_CUDA;
 }
 
-constexpr int kProfGroups = 9;
+constexpr int kProfGroups = 10;
 
 // Returns the record index, or -1 when profiling is off.
 int prof_begin(gnn_ctx* c, int group, int launches, cudaStream_t st) {
@@ -231,6 +240,7 @@ cudaError_t set_all_attrs() {
   if ((e = set_smem_attr<TileKind::EdgeUpdate, H, BF>()) != cudaSuccess) return e;
   if ((e = set_smem_attr<TileKind::NodeUpdate, H, BF>()) != cudaSuccess) return e;
   if ((e = set_smem_attr<TileKind::Filter, H, BF>()) != cudaSuccess) return e;
+  if ((e = set_smem_attr<TileKind::Embed, H, BF>()) != cudaSuccess) return e;
   return set_smem_attr<TileKind::Classifier, H, BF>();
 }
 
@@ -249,7 +259,7 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
 #ifdef GNN_TRACE
   p.trace = ((int)K == c->trace_kind) ? c->trace : nullptr;
 #endif
-  static const int group[6] = {1, 2, 3, 4, 5, 8};   // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier, Filter
+  static const int group[7] = {1, 2, 3, 4, 5, 8, 9};   // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier, Filter, Embed
   const int pr = prof_begin(c, group[(int)K], 1, st);
   mlp_tile_kernel<K, H, BF><<<grid, kThreads, smem, st>>>(p);
   prof_end(c, pr, st);
@@ -380,6 +390,7 @@ const char* gnn_error_string(int code) {
     case GNN_ERR_CUDA: return "CUDA error";
     case GNN_ERR_INDEX_RANGE: return "edge endpoint out of range";
     case GNN_ERR_DEVICE_TIMEOUT: return "device pipeline wait timed out";
+    case GNN_ERR_CAPACITY: return "output buffer too small";
     default: return "unknown status";
   }
 }
@@ -715,6 +726,149 @@ int gnn_filter_edges(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
 
+int gnn_embed_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes) {
+  if (!ctx || !weights_host) return GNN_ERR_INVALID_ARG;
+  const int H = ctx->cfg.hidden, Fn = ctx->cfg.n_node_feat;
+  const bool bf = ctx->cfg.precision == GNN_PRECISION_BF16;
+  if (weights_bytes < (size_t)kHeaderBytes) return GNN_ERR_BAD_WEIGHTS;
+  const uint8_t* blob = (const uint8_t*)weights_host;
+  int32_t hdr[8];
+  float eps;
+  int64_t n_floats;
+  std::memcpy(hdr, blob, 32);
+  std::memcpy(&eps, blob + 32, 4);
+  std::memcpy(&n_floats, blob + 40, 8);
+  const int L = hdr[4], D = hdr[6];
+  if ((uint32_t)hdr[0] != kEmbedMagic || hdr[1] != 1 || hdr[2] != Fn || hdr[3] != H || L < 2 || L > 4 ||
+      hdr[5] != ctx->cfg.precision || D < 1 || D > kMaxEmbedDim || !(eps > 0.f))
+    return GNN_ERR_BAD_WEIGHTS;
+  const int64_t want = (int64_t)H * Fn + 3 * H + (int64_t)(L - 1) * (H * H + 3 * H) + (int64_t)D * H + D;
+  if (n_floats != want || weights_bytes != (size_t)kHeaderBytes + 4 * (size_t)want) return GNN_ERR_BAD_WEIGHTS;
+  const float* f = (const float*)(blob + kHeaderBytes);
+  std::vector<Layer> lay(L);
+  for (int l = 0; l < L; ++l) {
+    const int in = l == 0 ? Fn : H;
+    lay[l] = {f, f + (size_t)H * in, f + (size_t)H * in + H, f + (size_t)H * in + 2 * H, in};
+    f += (size_t)H * in + 3 * H;
+  }
+  const float* wout = f;                                  // [D, H] then b_out [D]
+  std::vector<std::vector<float>> centred(2 * L);
+  if (!bf)
+    for (int l = 0; l < L; ++l) {
+      centre_layer(lay[l].W, lay[l].b, H, lay[l].in, centred[2 * l], centred[2 * l + 1]);
+      lay[l].W = centred[2 * l].data();
+      lay[l].b = centred[2 * l + 1].data();
+    }
+  KernelPlan pl;
+  for (int l = 1; l < L; ++l) { pl.job_acc[pl.n_jobs] = 0; pl.job_mat[pl.n_jobs] = l - 1; ++pl.n_jobs; }
+  for (int k = 0; k < Fn; ++k)                        // first-layer weight, transposed
+    for (int i = 0; i < H; ++i) pl.vecs.push_back(lay[0].W[(size_t)i * Fn + k]);
+  for (int l = 0; l < L; ++l) { push(pl.vecs, lay[l].b, H); push(pl.vecs, lay[l].g, H); push(pl.vecs, lay[l].be, H); }
+  push(pl.vecs, wout, (size_t)D * H + D);
+  finish_vecs(pl.vecs, H);
+  std::vector<uint8_t> packed((size_t)ctx->mat_bytes * (L - 1));
+  for (int l = 1; l < L; ++l) pack_block(lay[l].W, H, 0, H, !bf, packed.data() + (size_t)(l - 1) * ctx->mat_bytes);
+  if (ctx->embed_plan.d_vecs) { cudaFree(ctx->embed_plan.d_vecs); ctx->embed_plan.d_vecs = nullptr; }
+  if (ctx->d_embed_mats) { cudaFree(ctx->d_embed_mats); ctx->d_embed_mats = nullptr; }
+  ctx->embed_layers = 0;
+  cudaError_t err = dev_alloc((void**)&ctx->d_embed_mats, packed.size());
+  if (err == cudaSuccess) err = cudaMemcpy(ctx->d_embed_mats, packed.data(), packed.size(), cudaMemcpyHostToDevice);
+  if (err == cudaSuccess) err = dev_alloc((void**)&pl.d_vecs, pl.vecs.size() * 4);
+  if (err == cudaSuccess) err = cudaMemcpy(pl.d_vecs, pl.vecs.data(), pl.vecs.size() * 4, cudaMemcpyHostToDevice);
+  if (err != cudaSuccess) {
+    if (pl.d_vecs) cudaFree(pl.d_vecs);
+    if (ctx->d_embed_mats) { cudaFree(ctx->d_embed_mats); ctx->d_embed_mats = nullptr; }
+    return cuda_fail(err);
+  }
+  pl.wmats = ctx->d_embed_mats;
+  ctx->embed_plan = std::move(pl);
+  ctx->embed_layers = L;
+  ctx->embed_dim = D;
+  ctx->embed_eps = eps;
+  return GNN_OK;
+}
+
+int gnn_embed(gnn_ctx* ctx, const float* node_feats, int64_t n_nodes, float* embedding, gnn_stream_t stream) {
+  if (!ctx || n_nodes < 0 || n_nodes >= INT32_MAX || ctx->embed_layers == 0) return GNN_ERR_INVALID_ARG;
+  if (n_nodes == 0) return GNN_OK;
+  if (!node_feats || !embedding) return GNN_ERR_INVALID_ARG;
+  TileParams p{};
+  p.n_rows = (int)n_nodes;
+  p.n_nodes = (int)n_nodes;
+  p.n_layers = ctx->embed_layers;
+  p.n_feat = ctx->cfg.n_node_feat;
+  p.eps = ctx->embed_eps;
+  p.x = node_feats;
+  p.x_stride = ctx->cfg.n_node_feat;
+  p.emb = embedding;
+  p.emb_dim = ctx->embed_dim;
+  p.err = ctx->d_err;
+  cudaStream_t st = (cudaStream_t)stream;
+  const bool bf = ctx->cfg.precision == GNN_PRECISION_BF16;
+  if (ctx->cfg.hidden == 128) {
+    if (bf) launch_tile<TileKind::Embed, 128, true>(ctx, ctx->embed_plan, p, st);
+    else launch_tile<TileKind::Embed, 128, false>(ctx, ctx->embed_plan, p, st);
+  } else {
+    if (bf) launch_tile<TileKind::Embed, 64, true>(ctx, ctx->embed_plan, p, st);
+    else launch_tile<TileKind::Embed, 64, false>(ctx, ctx->embed_plan, p, st);
+  }
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
+
+int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const float* node_feats, int64_t n_nodes,
+                    float radius, int64_t max_edges, int32_t* edge_index, int32_t* n_edges, gnn_stream_t stream) {
+  if (!ctx || n_nodes < 0 || n_nodes >= INT32_MAX || emb_dim < 1 || emb_dim > kMaxEmbedDim || !(radius > 0.f) ||
+      max_edges < 0 || max_edges >= INT32_MAX || !n_edges)
+    return GNN_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (n_nodes == 0) {
+    const cudaError_t err = cudaMemsetAsync(n_edges, 0, sizeof(int32_t), st);
+    return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+  }
+  if (!embedding || !node_feats || (max_edges > 0 && !edge_index)) return GNN_ERR_INVALID_ARG;
+  const int N = (int)n_nodes, tb = 256;
+  const int grid = frnn_grid(radius);
+  const int n_cells = grid * grid * grid;
+  const int tiles = (N + kRadixTile - 1) / kRadixTile;
+  const size_t need = 5 * (size_t)N + 256 * (size_t)tiles + (size_t)n_cells + 1;
+  if (need > ctx->aux_ints) {
+    if (ctx->aux) { cudaStreamSynchronize(st); cudaFree(ctx->aux); ctx->aux = nullptr; ctx->aux_ints = 0; }
+    const cudaError_t err = dev_alloc((void**)&ctx->aux, need * sizeof(int));
+    if (err != cudaSuccess) return cuda_fail(err);
+    ctx->aux_ints = need;
+  }
+  int* keys_a = ctx->aux;
+  int* keys_b = keys_a + N;
+  int* vals_a = keys_b + N;
+  int* vals_b = vals_a + N;
+  int* counts = vals_b + N;
+  int* hist = counts + N;
+  int* cell_start = hist + 256 * (size_t)tiles;
+  frnn_cell_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(embedding, N, emb_dim, grid, keys_a, vals_a);
+  int bits = 0;
+  while (bits < 31 && ((n_cells - 1) >> bits) != 0) ++bits;
+  const int passes = ((bits > 0 ? bits : 1) + 7) / 8;
+  int *kin = keys_a, *vin = vals_a, *kout = keys_b, *vout = vals_b;
+  for (int ps = 0; ps < passes; ++ps) {
+    radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, N, 8 * ps, tiles, hist);
+    radix_offsets_kernel<<<1, 256, 0, st>>>(hist, tiles);
+    radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, N, 8 * ps, tiles, hist);
+    int* t = kin; kin = kout; kout = t;
+    t = vin; vin = vout; vout = t;
+  }
+  csr_rowptr_kernel<<<(n_cells + 1 + tb - 1) / tb, tb, 0, st>>>(kin, N, n_cells, cell_start);
+  const float r2 = radius * radius;
+  const int nb = (N + tb - 1) / tb;
+  frnn_pairs_kernel<<<nb, tb, 0, st>>>(embedding, node_feats, ctx->cfg.n_node_feat, N, emb_dim, r2, grid, kin, vin,
+                                       cell_start, 0, counts, nullptr, 0, nullptr, ctx->d_err);
+  compact_scan_kernel<<<1, 1024, 0, st>>>(counts, N, n_edges);
+  frnn_pairs_kernel<<<nb, tb, 0, st>>>(embedding, node_feats, ctx->cfg.n_node_feat, N, emb_dim, r2, grid, kin, vin,
+                                       cell_start, 1, counts, n_edges, (int)max_edges, edge_index, ctx->d_err);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? GNN_OK : cuda_fail(err);
+}
+
 int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge_index, int64_t n_nodes,
                      int64_t n_edges, float threshold, int32_t* labels, gnn_stream_t stream) {
   if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX) return GNN_ERR_INVALID_ARG;
@@ -785,6 +939,7 @@ int gnn_status(gnn_ctx* ctx, gnn_stream_t stream) {
   if (err == cudaSuccess) err = cudaMemset(ctx->d_err, 0, 4);
   if (err != cudaSuccess) return cuda_fail(err);
   if (word & DEV_ERR_TIMEOUT) return GNN_ERR_DEVICE_TIMEOUT;
+  if (word & DEV_ERR_CAPACITY) return GNN_ERR_CAPACITY;
   if (word & DEV_ERR_INDEX_RANGE) return GNN_ERR_INDEX_RANGE;
   return GNN_OK;
 }
@@ -798,6 +953,9 @@ void gnn_destroy(gnn_ctx* ctx) {
     if (ctx->plan[i].d_vecs) cudaFree(ctx->plan[i].d_vecs);
   if (ctx->filter_plan.d_vecs) cudaFree(ctx->filter_plan.d_vecs);
   if (ctx->d_filter_mats) cudaFree(ctx->d_filter_mats);
+  if (ctx->embed_plan.d_vecs) cudaFree(ctx->embed_plan.d_vecs);
+  if (ctx->d_embed_mats) cudaFree(ctx->d_embed_mats);
+  if (ctx->aux) cudaFree(ctx->aux);
   if (ctx->d_err) cudaFree(ctx->d_err);
   if (ctx->stage) cudaFree(ctx->stage);
   for (auto& r : ctx->prof) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }

@@ -45,7 +45,10 @@ enum class TileKind : int {
   NodeUpdate  = 3,     // h <- MLP_node([h, sum of incoming e]); then P_s, P_d of new h
   Classifier  = 4,     // score = sigmoid(w_o . MLP_cls([h_src, h_dst, e]) + b_o)
   Filter      = 5,     // filtering step: score = sigmoid(w_o . MLP_f([x_src, x_dst]) + b_o), input edge order
+  Embed       = 6,     // embedding step: y = normalize(W_out . MLP_emb(x) + b_out), D outputs per hit
 };
+
+constexpr int kMaxEmbedDim = 16;
 
 constexpr int kThreads = 640;
 // Register split (setmaxnreg): launch at 96 per thread (640 threads x 96 = 61440);
@@ -89,6 +92,8 @@ struct TileParams {
   float* scores;              // [E] input order
   uint32_t* err;              // device error word
   const int32_t* ei_in;       // filter: [2, E] input edge index (rows in input order)
+  float* emb;                 // embedding: [N, emb_dim] output
+  int emb_dim;
 #ifdef GNN_TRACE
   unsigned long long* trace;  // [3 roles][kTraceEvents] %globaltimer stamps of CTA 0
 #endif
@@ -726,6 +731,69 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           const float* vl = vb + 3 * (L - 1) * H;
           const bool w0 = ok && ok0, w1 = ok && ok1;
           ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { store_t16_chunk(p.e, row0, w0, w1, k, t); });
+        }
+      } else if constexpr (KIND == TileKind::Embed) {
+        // vec layout: [W1^T (F_n x H), (b_l, gamma_l, beta_l) for l = 1..L, W_out rows (D x H), b_out (D)]
+        // L hidden layers (layer 1 on CUDA cores), then the D outputs on CUDA cores, L2-normalised.
+#pragma unroll
+        for (int i = 0; i < 4 * NB; ++i) v[i] = 0.f;
+        for (int k = 0; k < p.n_feat; ++k) {
+          const float x0 = ok0 ? p.x[(size_t)row0 * p.x_stride + k] : 0.f;
+          const float x1 = ok1 ? p.x[(size_t)row1 * p.x_stride + k] : 0.f;
+#pragma unroll
+          for (int b = 0; b < NB; b += 2) {
+            const float4 w = vq4(vecs + k * H, b);
+            v[4 * b] = fmaf(w.x, x0, v[4 * b]); v[4 * b + 1] = fmaf(w.y, x0, v[4 * b + 1]);
+            v[4 * b + 2] = fmaf(w.x, x1, v[4 * b + 2]); v[4 * b + 3] = fmaf(w.y, x1, v[4 * b + 3]);
+            v[4 * b + 4] = fmaf(w.z, x0, v[4 * b + 4]); v[4 * b + 5] = fmaf(w.w, x0, v[4 * b + 5]);
+            v[4 * b + 6] = fmaf(w.z, x1, v[4 * b + 6]); v[4 * b + 7] = fmaf(w.w, x1, v[4 * b + 7]);
+          }
+        }
+        const float* vb = vecs + p.n_feat * H;
+        add_vec(v, vb);
+        ln_relu(v, vb + H, vb + 2 * H);
+        for (int l = 2; l <= L; ++l) {
+          put_a(v);
+          arrive_a(j, seq); next_job();
+          wait_job();
+          load_d(v);
+          const float* vl = vb + 3 * (l - 1) * H;
+          add_vec(v, vl);
+          ln_relu(v, vl + H, vl + 2 * H);
+        }
+        if constexpr (BF) {                  // the projection's input is a bf16 activation
+#pragma unroll
+          for (int i = 0; i < 4 * NB; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+        }
+        const float* wout = vb + 3 * L * H;
+        float y0[kMaxEmbedDim], y1[kMaxEmbedDim];
+        float n0 = 0.f, n1 = 0.f;
+        for (int d = 0; d < p.emb_dim; ++d) {
+          float z0 = 0.f, z1 = 0.f;
+#pragma unroll
+          for (int k = 0; k < NB; k += 2) {
+            const float4 w = vq4(wout + d * H, k);
+            z0 = fmaf(v[4 * k], w.x, fmaf(v[4 * k + 1], w.y, fmaf(v[4 * k + 4], w.z, fmaf(v[4 * k + 5], w.w, z0))));
+            z1 = fmaf(v[4 * k + 2], w.x, fmaf(v[4 * k + 3], w.y, fmaf(v[4 * k + 6], w.z, fmaf(v[4 * k + 7], w.w, z1))));
+          }
+          const float bo = wout[p.emb_dim * H + d];
+          z0 = quad_sum(z0) + bo;
+          z1 = quad_sum(z1) + bo;
+#pragma unroll
+          for (int i = 0; i < kMaxEmbedDim; ++i)
+            if (i == d) { y0[i] = z0; y1[i] = z1; }
+          n0 = fmaf(z0, z0, n0);
+          n1 = fmaf(z1, z1, n1);
+        }
+        const float i0 = n0 > 0.f ? rsqrtf(n0) : 0.f, i1 = n1 > 0.f ? rsqrtf(n1) : 0.f;
+        if (ok && (lane & 3) == 0) {
+#pragma unroll
+          for (int i = 0; i < kMaxEmbedDim; ++i) {
+            if (i < p.emb_dim) {
+              if (ok0) p.emb[(size_t)row0 * p.emb_dim + i] = y0[i] * i0;
+              if (ok1) p.emb[(size_t)row1 * p.emb_dim + i] = y1[i] * i1;
+            }
+          }
         }
       } else if constexpr (KIND == TileKind::Filter) {
         // vec layout: [W1^T (2 F_n x H), b1, gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]

@@ -13,6 +13,7 @@ namespace gnn {
 enum : uint32_t {
   DEV_ERR_INDEX_RANGE = 1u,   // an edge endpoint was outside [0, n_nodes)
   DEV_ERR_TIMEOUT     = 2u,   // a bounded wait expired (pipeline stalled)
+  DEV_ERR_CAPACITY    = 4u,   // an output buffer was too small (graph building)
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

@@ -334,3 +334,44 @@ def pack_filter_blob(cfg: ModelConfig, fw: dict) -> bytes:
                          cfg.precision, 0, 0, cfg.ln_eps, 0, len(payload) // 4)
     return header + payload
 
+
+# --------------------------------------------------------------------------- embedding MLP
+
+EMBED_MAGIC = 0x4D454E47  # "GNEM" little-endian
+
+
+def init_embed_weights(cfg: ModelConfig, dim: int = 8, seed: int = 2) -> dict:
+    """Random-init embedding MLP: mlp_layers hidden layers on x (n_node_feat inputs) drawn as in
+    init_weights, then W_out [dim, H] ~ N(0, 1/H) and b_out ~ N(0, 0.1^2); bf16-rounded for the
+    bf16 model."""
+    rng = np.random.default_rng(seed)
+    H = cfg.hidden
+    fan_in = cfg.n_node_feat
+    layers = []
+    for _ in range(cfg.mlp_layers):
+        W = (rng.standard_normal((H, fan_in)) / np.sqrt(fan_in)).astype(np.float32)
+        b = (0.1 * rng.standard_normal(H)).astype(np.float32)
+        g = (1.0 + 0.1 * rng.standard_normal(H)).astype(np.float32)
+        be = (0.1 * rng.standard_normal(H)).astype(np.float32)
+        layers.append((W, b, g, be))
+        fan_in = H
+    out = {"layers": layers, "out_w": (rng.standard_normal((dim, H)) / np.sqrt(H)).astype(np.float32),
+           "out_b": (0.1 * rng.standard_normal(dim)).astype(np.float32)}
+    if cfg.precision == PRECISION_BF16:
+        out = {"layers": [tuple(_round_bf16(t) for t in lay) for lay in layers],
+               "out_w": _round_bf16(out["out_w"]), "out_b": _round_bf16(out["out_b"])}
+    return out
+
+
+def pack_embed_blob(cfg: ModelConfig, ew: dict) -> bytes:
+    """Embedding blob: 8 int32 (magic, version 1, n_node_feat, hidden, layers, precision, dim, 0),
+    float32 ln_eps, int32 0, int64 float count; per layer W, b, gamma, beta; W_out [dim, H], b_out."""
+    arrays = []
+    for (W, b, g, be) in ew["layers"]:
+        arrays += [W, b, g, be]
+    arrays += [ew["out_w"], ew["out_b"]]
+    payload = b"".join(np.ascontiguousarray(a, dtype="<f4").tobytes() for a in arrays)
+    header = struct.pack("<8i f i q", EMBED_MAGIC, 1, cfg.n_node_feat, cfg.hidden, len(ew["layers"]),
+                         cfg.precision, ew["out_w"].shape[0], 0, cfg.ln_eps, 0, len(payload) // 4)
+    return header + payload
+

@@ -455,3 +455,44 @@ def test_apply_filtering_keeps_order_and_drops_nan():
     kept, ids = O.apply_filtering(sc, ei, 0.5)
     assert ids.tolist() == [0, 3]
     assert kept.tolist() == [[0, 3], [5, 8]]
+
+
+# ------------------------------------------------------------- embedding and graph building
+
+def test_embed_is_unit_length_and_matches_hand_layer():
+    ew = {"layers": [(np.array([[1.0, -0.5], [0.25, 2.0]]), np.array([0.1, 0.0]), np.array([1.0, 1.0]),
+                      np.array([0.0, 0.3]))],
+          "out_w": np.array([[1.0, 2.0], [-1.0, 0.5], [0.0, 1.0]]), "out_b": np.array([0.1, 0.0, -0.2])}
+    x = np.array([[0.3, 0.7], [-1.0, 0.2]], np.float32)
+    y = O.embed(ew, x, HAND_EPS)
+    for k in range(2):
+        a, b = float(x[k, 0]), float(x[k, 1])
+        h = _relu2(_ln2(a - 0.5 * b + 0.1, 0.25 * a + 2.0 * b, (1.0, 1.0), (0.0, 0.3)))
+        z = np.array([h[0] + 2 * h[1] + 0.1, -h[0] + 0.5 * h[1], h[1] - 0.2])
+        np.testing.assert_allclose(y[k], z / np.linalg.norm(z), atol=1e-12)
+    np.testing.assert_allclose(np.linalg.norm(y, axis=1), 1.0, atol=1e-12)
+
+
+def test_radius_graph_against_brute_force_and_kdtree():
+    rng = np.random.default_rng(11)
+    emb = rng.standard_normal((400, 5)).astype(np.float32)
+    emb /= np.linalg.norm(emb, axis=1, keepdims=True)
+    r_col = rng.integers(0, 4, 400).astype(np.float32)          # layer-like radii with many ties
+    radius = 0.45
+    got = O.radius_graph(emb, r_col, radius)
+    want = []
+    for i in range(400):                                         # float64 brute force, away from the boundary
+        for j in range(i + 1, 400):
+            d2 = float(((emb[i].astype(np.float64) - emb[j]) ** 2).sum())
+            if d2 < radius * radius:
+                a, b = (i, j) if (r_col[i] < r_col[j] or (r_col[i] == r_col[j] and i < j)) else (j, i)
+                want.append((a, b))
+    assert len(want) > 200
+    got_set, want_set = set(map(tuple, got.tolist())), set(want)
+    diff = got_set ^ want_set
+    for a, b in diff:                                            # only pairs on the boundary may differ
+        d2 = float(((emb[a].astype(np.float64) - emb[b]) ** 2).sum())
+        assert abs(d2 - radius * radius) < 1e-5
+    kd = pytest.importorskip("scipy.spatial")
+    cand = np.array(sorted(kd.cKDTree(emb.astype(np.float64)).query_pairs(radius * 1.001)), np.int64)
+    np.testing.assert_array_equal(O.radius_graph(emb, r_col, radius, cand), got)
