@@ -4,16 +4,24 @@
 //
 // The embeddings are unit vectors, so each coordinate lies in [-1, 1].  Hits
 // are binned on a uniform grid over their first three coordinates with cells
-// wider than the radius (a coordinate outside [-1, 1] is clamped to the edge
-// cells, which keeps the search exact, only slower), and sorted by cell (the library's stable radix
-// sort).  Each hit then visits the 27 cells around its own and tests the full
-// D-dimensional squared distance, summed over the coordinates in order with one
-// rounding per product and per sum (no fused multiply-add), against radius^2
-// rounded to fp32.  A pair is found once, by its hit with the smaller index,
-// and oriented from the hit with the smaller r (column 0 of the node features,
-// index as tie-break) to the other.  A counting pass, a scan and a writing pass
-// make the output order deterministic: by the finding hit's position in the
-// cell order, then by cell and position of the partner.
+// a little wider than half the radius (a coordinate outside [-1, 1] is clamped
+// to the edge cells, which keeps the search exact, only slower), and sorted by
+// cell (the library's stable radix sort); their embeddings and r values are
+// then gathered into that order, zero-padded to a multiple of four
+// coordinates.  A pair within the radius lies at most two cells apart on each
+// axis, so the partners of a hit sit in the 5 x 5 "rows" of cells around its
+// own, and in each row in one run of at most five consecutive cells, which is
+// one contiguous range of sorted positions.  Rows before the hit's own row hold
+// only earlier positions: each pair is visited once, by its earlier sorted
+// position, which scans 13 rows (its own row from the next position on).
+//
+// The test is the full squared distance, summed over the coordinates in order
+// with one rounding per product and per sum (no fused multiply-add; the zero
+// padding adds exact zeros), against radius^2 rounded to fp32.  Each pair
+// becomes one edge, oriented from the hit with the smaller r (column 0 of the
+// node features, hit id as tie-break).  A counting pass, a scan and a writing
+// pass make the output order deterministic: by the visiting hit's sorted
+// position, then by row and position of the partner.
 #pragma once
 #include <cstdint>
 #include "ptx.cuh"
@@ -21,11 +29,12 @@
 namespace gnn {
 
 constexpr int kFrnnMaxGrid = 128;        // cells per axis
+constexpr int kFrnnReach = 2;            // cells a partner can lie away on each axis
 
-// Cells per axis: cells a little wider than the radius (0.1 % margin), so that the rounding of the
-// cell coordinates and of the distance test never puts a pair within the radius two cells apart.
+// Cells per axis: cells 0.1 % wider than half the radius, so that the rounding of the cell
+// coordinates and of the distance test never puts a pair within the radius three cells apart.
 __host__ __device__ inline int frnn_grid(float radius) {
-  const float cells = 1.998f / radius;
+  const float cells = 1.998f * (float)kFrnnReach / radius;
   return cells >= (float)kFrnnMaxGrid ? kFrnnMaxGrid : (cells < 1.0f ? 1 : (int)cells);
 }
 
@@ -46,22 +55,41 @@ __global__ void frnn_cell_kernel(const float* __restrict__ emb, int n, int dim, 
   vals[i] = i;
 }
 
-// One thread per sorted position t (hit i = ids[t]).  write == 0: counts[t] = pairs found by i;
-// write == 1: those pairs at offsets[t] (exclusive scan of counts), when the total fits.
-__global__ void frnn_pairs_kernel(const float* __restrict__ emb, const float* __restrict__ x, int x_stride, int n,
-                                  int dim, float r2, int grid, const int* __restrict__ cell_keys,
-                                  const int* __restrict__ ids, const int* __restrict__ cell_start, int write,
-                                  int* __restrict__ counts, const int* __restrict__ total, int capacity,
-                                  int32_t* __restrict__ out, uint32_t* err) {
+// Sorted copies: emb_s [n, 4 * CH] (zero-padded), r_s [n] = x[ids[t], 0].
+template <int CH>
+__global__ void frnn_gather_kernel(const float* __restrict__ emb, const float* __restrict__ x, int x_stride, int n,
+                                   int dim, const int* __restrict__ ids, float4* __restrict__ emb_s,
+                                   float* __restrict__ r_s) {
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= n) return;
   const int i = ids[t];
-  float ei[16];
+  const float* e = emb + (size_t)i * dim;
 #pragma unroll
-  for (int d = 0; d < 16; ++d) ei[d] = d < dim ? emb[(size_t)i * dim + d] : 0.f;
-  const int key = cell_keys[t];
-  const int c2 = key % grid, c1 = (key / grid) % grid, c0 = key / (grid * grid);
-  int found = 0, pos = 0, n_total = 0;
+  for (int c = 0; c < CH; ++c) {
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = 4 * c + k < dim ? e[4 * c + k] : 0.f;
+    emb_s[(size_t)t * CH + c] = make_float4(v[0], v[1], v[2], v[3]);
+  }
+  r_s[t] = x[(size_t)i * x_stride];
+}
+
+__device__ __forceinline__ float frnn_acc(float s, float a, float b) {
+  const float d = a - b;
+  return __fadd_rn(s, __fmul_rn(d, d));
+}
+
+// One thread per sorted position t.  write == 0: counts[t] = pairs visited from t;
+// write == 1: those pairs at offsets[t] (exclusive scan of counts), when the total fits.
+template <int CH>
+__global__ void __launch_bounds__(256) frnn_pairs_kernel(
+    const float4* __restrict__ emb_s, const float* __restrict__ r_s, int n, float r2, int grid,
+    const int* __restrict__ cell_keys, const int* __restrict__ ids, const int* __restrict__ cell_start, int write,
+    int* __restrict__ counts, const int* __restrict__ total, int capacity, int32_t* __restrict__ out,
+    uint32_t* err) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= n) return;
+  int pos = 0, n_total = 0;
   if (write) {
     n_total = *total;
     if (n_total > capacity) {
@@ -70,36 +98,47 @@ __global__ void frnn_pairs_kernel(const float* __restrict__ emb, const float* __
     }
     pos = counts[t];
   }
-  const float ri = write ? x[(size_t)i * x_stride] : 0.f;
-  for (int a = c0 - 1; a <= c0 + 1; ++a) {
-    if (a < 0 || a >= grid) continue;
-    for (int b = c1 - 1; b <= c1 + 1; ++b) {
-      if (b < 0 || b >= grid) continue;
-      for (int c = c2 - 1; c <= c2 + 1; ++c) {
-        if (c < 0 || c >= grid) continue;
-        const int cell = (a * grid + b) * grid + c;
-        for (int q = cell_start[cell], q1 = cell_start[cell + 1]; q < q1; ++q) {
-          const int j = ids[q];
-          if (j <= i) continue;
-          const float* ej = emb + (size_t)j * dim;
-          float s = 0.f;                       // no fused multiply-add: one rounding per product and sum
+  float4 q[CH];
 #pragma unroll
-          for (int d = 0; d < 16; ++d) {
-            if (d < dim) {
-              const float diff = ei[d] - ej[d];
-              s = __fadd_rn(s, __fmul_rn(diff, diff));
-            }
-          }
-          if (!(s < r2)) continue;
-          if (write) {
-            const float rj = x[(size_t)j * x_stride];
-            const bool i_first = ri < rj || (ri == rj && i < j);
-            out[pos] = i_first ? i : j;
-            out[(size_t)n_total + pos] = i_first ? j : i;
-            ++pos;
-          } else {
-            ++found;
-          }
+  for (int c = 0; c < CH; ++c) q[c] = emb_s[(size_t)t * CH + c];
+  const int key = cell_keys[t];
+  const int c2 = key % grid, c1 = (key / grid) % grid, c0 = key / (grid * grid);
+  const int lo2 = c2 - kFrnnReach < 0 ? 0 : c2 - kFrnnReach;
+  const int hi2 = c2 + kFrnnReach >= grid ? grid - 1 : c2 + kFrnnReach;
+  int i = 0;
+  float ri = 0.f;
+  if (write) { i = ids[t]; ri = r_s[t]; }
+  int found = 0;
+  for (int a = 0; a <= kFrnnReach; ++a) {
+    const int ra = c0 + a;
+    if (ra >= grid) break;
+    for (int b = (a == 0 ? 0 : -kFrnnReach); b <= kFrnnReach; ++b) {
+      const int rb = c1 + b;
+      if (rb < 0 || rb >= grid) continue;
+      const int row = (ra * grid + rb) * grid;
+      int p = cell_start[row + lo2];
+      const int p1 = cell_start[row + hi2 + 1];
+      if (a == 0 && b == 0) p = t + 1;
+      for (; p < p1; ++p) {
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < CH; ++c) {
+          const float4 e = emb_s[(size_t)p * CH + c];
+          s = frnn_acc(s, q[c].x, e.x);
+          s = frnn_acc(s, q[c].y, e.y);
+          s = frnn_acc(s, q[c].z, e.z);
+          s = frnn_acc(s, q[c].w, e.w);
+        }
+        if (!(s < r2)) continue;
+        if (write) {
+          const int j = ids[p];
+          const float rj = r_s[p];
+          const bool i_first = ri < rj || (ri == rj && i < j);
+          out[pos] = i_first ? i : j;
+          out[(size_t)n_total + pos] = i_first ? j : i;
+          ++pos;
+        } else {
+          ++found;
         }
       }
     }

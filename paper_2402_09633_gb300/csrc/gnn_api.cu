@@ -831,21 +831,27 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   const int grid = frnn_grid(radius);
   const int n_cells = grid * grid * grid;
   const int tiles = (N + kRadixTile - 1) / kRadixTile;
-  const size_t need = 5 * (size_t)N + 256 * (size_t)tiles + (size_t)n_cells + 1;
+  const int chunks = (emb_dim + 3) / 4;                   // float4 chunks per sorted embedding
+  // scratch: emb_s [N, 4 * chunks] (first, 16-byte aligned), r_s, keys/vals (two buffers each),
+  // per-hit counts, radix histograms, cell starts
+  const size_t need = 4 * (size_t)chunks * N + 6 * (size_t)N + 256 * (size_t)tiles + (size_t)n_cells + 1;
   if (need > ctx->aux_ints) {
     if (ctx->aux) { cudaStreamSynchronize(st); cudaFree(ctx->aux); ctx->aux = nullptr; ctx->aux_ints = 0; }
     const cudaError_t err = dev_alloc((void**)&ctx->aux, need * sizeof(int));
     if (err != cudaSuccess) return cuda_fail(err);
     ctx->aux_ints = need;
   }
-  int* keys_a = ctx->aux;
+  float4* emb_s = (float4*)ctx->aux;
+  float* r_s = (float*)(ctx->aux + 4 * (size_t)chunks * N);
+  int* keys_a = (int*)(r_s + N);
   int* keys_b = keys_a + N;
   int* vals_a = keys_b + N;
   int* vals_b = vals_a + N;
   int* counts = vals_b + N;
   int* hist = counts + N;
   int* cell_start = hist + 256 * (size_t)tiles;
-  frnn_cell_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(embedding, N, emb_dim, grid, keys_a, vals_a);
+  const int nb = (N + tb - 1) / tb;
+  frnn_cell_kernel<<<nb, tb, 0, st>>>(embedding, N, emb_dim, grid, keys_a, vals_a);
   int bits = 0;
   while (bits < 31 && ((n_cells - 1) >> bits) != 0) ++bits;
   const int passes = ((bits > 0 ? bits : 1) + 7) / 8;
@@ -859,12 +865,23 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   }
   csr_rowptr_kernel<<<(n_cells + 1 + tb - 1) / tb, tb, 0, st>>>(kin, N, n_cells, cell_start);
   const float r2 = radius * radius;
-  const int nb = (N + tb - 1) / tb;
-  frnn_pairs_kernel<<<nb, tb, 0, st>>>(embedding, node_feats, ctx->cfg.n_node_feat, N, emb_dim, r2, grid, kin, vin,
-                                       cell_start, 0, counts, nullptr, 0, nullptr, ctx->d_err);
-  compact_scan_kernel<<<1, 1024, 0, st>>>(counts, N, n_edges);
-  frnn_pairs_kernel<<<nb, tb, 0, st>>>(embedding, node_feats, ctx->cfg.n_node_feat, N, emb_dim, r2, grid, kin, vin,
-                                       cell_start, 1, counts, n_edges, (int)max_edges, edge_index, ctx->d_err);
+  const int xs = ctx->cfg.n_node_feat;
+  switch (chunks) {
+#define GNN_FRNN_CASE(CH)                                                                                        \
+  case CH:                                                                                                       \
+    frnn_gather_kernel<CH><<<nb, tb, 0, st>>>(embedding, node_feats, xs, N, emb_dim, vin, emb_s, r_s);         \
+    frnn_pairs_kernel<CH><<<nb, tb, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, 0, counts, nullptr, \
+                                             0, nullptr, ctx->d_err);                                           \
+    compact_scan_kernel<<<1, 1024, 0, st>>>(counts, N, n_edges);                                                 \
+    frnn_pairs_kernel<CH><<<nb, tb, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, 1, counts, n_edges, \
+                                             (int)max_edges, edge_index, ctx->d_err);                           \
+    break;
+    GNN_FRNN_CASE(1)
+    GNN_FRNN_CASE(2)
+    GNN_FRNN_CASE(3)
+    GNN_FRNN_CASE(4)
+#undef GNN_FRNN_CASE
+  }
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
