@@ -4,7 +4,10 @@
 One step = one gnn_infer call on one synthetic full event (300,000 nodes,
 1,000,000 candidate edges, 12 node features, H=128, T=8, 3-layer MLPs):
 device-side CSR build, encoders, eight message-passing iterations and the
-classifier, inputs resident in HBM.  Prints one JSON line (rank 0).
+classifier, inputs resident in HBM.  Prints one JSON line (rank 0).  After the
+timed steps, `pipeline` times every stage of the tracking pipeline once more on
+the same event (embedding, graph building, filtering, the network, track
+labels); those stages are outside `value`.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
 
@@ -245,6 +248,47 @@ def whole_job(local_s: float, local_units: float, world: int, device=None):
 
 
 # ------------------------------------------------------------------ GB300 arm
+def run_pipeline(net, w: S.Workload, x, dev, reps: int = 5):
+    """Every stage of the tracking pipeline on the bench event, each timed with CUDA events on the
+    current stream (mean of `reps` after one untimed call): embedding, fixed-radius graph building,
+    filtering, the interaction network on the kept edges, track labels.  Random-init embedding and
+    filter weights; the radius is the median distance to the 4th nearest neighbour of 2,000 sampled
+    hits, the filter threshold the median filter score (setup, outside the timed calls)."""
+    import torch
+    net.load_embedding(S.pack_embed_blob(w.model, S.init_embed_weights(w.model, 8, 2)))
+    net.load_filter(S.pack_filter_blob(w.model, S.init_filter_weights(w.model, 1)))
+    N = x.shape[0]
+    out = {}
+
+    def timed(name, fn):
+        res = fn()
+        torch.cuda.synchronize(dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            res = fn()
+        b.record()
+        torch.cuda.synchronize(dev)
+        out[name + "_ms"] = a.elapsed_time(b) / reps
+        return res
+
+    emb = timed("embed", lambda: net.embed(x))
+    sample = emb[torch.randperm(N, generator=torch.Generator().manual_seed(0))[:2000].to(dev)]
+    radius = float(torch.cdist(sample, emb).kthvalue(5, dim=1).values.median())
+    cand, n_cand = timed("build_graph", lambda: net.build_graph(emb, x, radius, 40 * N))
+    cand = cand.contiguous()
+    fsc, _, _ = net.filter_edges(x, cand, 0.5)
+    thr = float(fsc.median())
+    _, kept, _ = timed("filter", lambda: net.filter_edges(x, cand, thr))
+    kept = kept.contiguous()
+    scores = timed("infer", lambda: net.infer(x, kept))
+    timed("track_labels", lambda: net.track_labels(scores, kept, N, 0.5))
+    out.update({"total_ms": sum(v for k, v in out.items() if k.endswith("_ms")), "n_hits": N,
+                "embedding_dim": 8, "radius": radius, "candidate_edges": n_cand,
+                "filter_threshold": thr, "kept_edges": int(kept.shape[1]), "device_status": net.status()})
+    return out
+
+
 def run_gb300(args, rank: int, world: int, local: int):
     import torch
     import torch.distributed as dist
@@ -326,6 +370,8 @@ def run_gb300(args, rank: int, world: int, local: int):
             dist.destroy_process_group()
         return
 
+    pipeline = run_pipeline(net, w, x, dev) if w.n_events == 1 else None
+
     peaks, peak_src = load_peaks()
     model = step_model(w)
     groups = {g: {"ms_total": ms, "launches": n} for g, (ms, n) in prof.items() if n}
@@ -364,6 +410,7 @@ def run_gb300(args, rank: int, world: int, local: int):
             "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms,
                               "bytes_alg": model["bytes"], "flops_alg": model["flops"]},
             "kernels": groups,
+            "pipeline": pipeline,
             "cpu_baseline": cpu,
             "e2e": {"value": job_edges / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": int(x_np.nbytes + ei_np.nbytes),
