@@ -77,6 +77,53 @@ __global__ void __launch_bounds__(1024) compact_scan_kernel(int* __restrict__ co
   if (t == 0) *total = carry > 0x7fffffffLL ? 0x7fffffff : (int)carry;
 }
 
+// Exclusive scan of a long int array in place, in three launches: scan_reduce_kernel (sum of
+// every 1024 entries, saturated at INT32_MAX), compact_scan_kernel over those sums (offsets and
+// the total), scan_apply_kernel (offset plus the scan inside each 1024 entries).  A total above
+// INT32_MAX saturates there; the offsets are then meaningless and the caller must not use them.
+constexpr int kScanBlock = 1024;
+
+__global__ void __launch_bounds__(kScanBlock) scan_reduce_kernel(const int* __restrict__ v, int n,
+                                                                 int* __restrict__ sums) {
+  __shared__ long long wsum[32];
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int i = blockIdx.x * kScanBlock + t;
+  long long x = i < n ? v[i] : 0;
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  if (lane == 0) wsum[warp] = x;
+  __syncthreads();
+  if (t == 0) {
+    long long s = 0;
+    for (int w = 0; w < 32; ++w) s += wsum[w];
+    sums[blockIdx.x] = s > 0x7fffffffLL ? 0x7fffffff : (int)s;
+  }
+}
+
+__global__ void __launch_bounds__(kScanBlock) scan_apply_kernel(int* __restrict__ v, int n,
+                                                                const int* __restrict__ offsets) {
+  __shared__ int wsum[32];
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int i = blockIdx.x * kScanBlock + t;
+  const int c = i < n ? v[i] : 0;
+  int x = c;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = wsum[lane];
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    wsum[lane] = w;
+  }
+  __syncthreads();
+  if (i < n) v[i] = offsets[blockIdx.x] + (warp > 0 ? wsum[warp - 1] : 0) + x - c;
+}
+
 __global__ void __launch_bounds__(kCompactThreads) compact_scatter_kernel(
     const float* __restrict__ scores, const int32_t* __restrict__ ei, int m, float threshold,
     const int* __restrict__ offsets, const int* __restrict__ total, int32_t* __restrict__ out_ei,

@@ -833,8 +833,9 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   const int tiles = (N + kRadixTile - 1) / kRadixTile;
   const int chunks = (emb_dim + 3) / 4;                   // float4 chunks per sorted embedding
   // scratch: emb_s [N, 4 * chunks] (first, 16-byte aligned), r_s, keys/vals (two buffers each),
-  // per-hit counts, radix histograms, cell starts
-  const size_t need = 4 * (size_t)chunks * N + 6 * (size_t)N + 256 * (size_t)tiles + (size_t)n_cells + 1;
+  // per-hit counts, per-block sums, radix histograms, cell starts
+  const int nb = (N + tb - 1) / tb;
+  const size_t need = 4 * (size_t)chunks * N + 6 * (size_t)N + (size_t)nb + 256 * (size_t)tiles + (size_t)n_cells + 1;
   if (need > ctx->aux_ints) {
     if (ctx->aux) { cudaStreamSynchronize(st); cudaFree(ctx->aux); ctx->aux = nullptr; ctx->aux_ints = 0; }
     const cudaError_t err = dev_alloc((void**)&ctx->aux, need * sizeof(int));
@@ -848,9 +849,9 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   int* vals_a = keys_b + N;
   int* vals_b = vals_a + N;
   int* counts = vals_b + N;
-  int* hist = counts + N;
+  int* block_sums = counts + N;
+  int* hist = block_sums + nb;
   int* cell_start = hist + 256 * (size_t)tiles;
-  const int nb = (N + tb - 1) / tb;
   frnn_cell_kernel<<<nb, tb, 0, st>>>(embedding, N, emb_dim, grid, keys_a, vals_a);
   int bits = 0;
   while (bits < 31 && ((n_cells - 1) >> bits) != 0) ++bits;
@@ -866,13 +867,16 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   csr_rowptr_kernel<<<(n_cells + 1 + tb - 1) / tb, tb, 0, st>>>(kin, N, n_cells, cell_start);
   const float r2 = radius * radius;
   const int xs = ctx->cfg.n_node_feat;
+  const int sb = (N + kScanBlock - 1) / kScanBlock;
   switch (chunks) {
 #define GNN_FRNN_CASE(CH)                                                                                        \
   case CH:                                                                                                       \
     frnn_gather_kernel<CH><<<nb, tb, 0, st>>>(embedding, node_feats, xs, N, emb_dim, vin, emb_s, r_s);         \
     frnn_pairs_kernel<CH><<<nb, tb, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, 0, counts, nullptr, \
                                              0, nullptr, ctx->d_err);                                           \
-    compact_scan_kernel<<<1, 1024, 0, st>>>(counts, N, n_edges);                                                 \
+    scan_reduce_kernel<<<sb, kScanBlock, 0, st>>>(counts, N, block_sums);                                      \
+    compact_scan_kernel<<<1, 1024, 0, st>>>(block_sums, sb, n_edges);                                            \
+    scan_apply_kernel<<<sb, kScanBlock, 0, st>>>(counts, N, block_sums);                                       \
     frnn_pairs_kernel<CH><<<nb, tb, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, 1, counts, n_edges, \
                                              (int)max_edges, edge_index, ctx->d_err);                           \
     break;
