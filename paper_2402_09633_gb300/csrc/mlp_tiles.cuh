@@ -203,9 +203,11 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         }
       }
       __syncwarp();
-      if (resident && (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier)) {
+      if (resident && KIND == TileKind::Classifier) {
         // L2 prefetcher: while the workers are on tile pair k, warm L2 with the
-        // edge-state tiles and the gathered P_s / P_d rows of pair k+1.
+        // edge-state tiles and the gathered P_s / P_d rows of pair k+1.  (The edge update
+        // prefetches from its workers instead: this warp made it 4 % slower, with only the
+        // gathered rows 7 %, with the rows paced to its layer-2 point 29 %.)
         const uint64_t t0 = global_timer_ns();
         for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
           const int prev = pair - (int)gridDim.x;
@@ -654,6 +656,15 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         for (int l = 2; l <= L; ++l) {
           wait_job();
           GNN_TRACE_W(5 + 2 * (l - 1));
+          if (KIND == TileKind::EdgeUpdate && l == 2 && ws == 0 && lane == 0) {
+            // Warm L2 with this slot's next edge-state tile, a few microseconds before its load
+            // (bulk prefetch: the copy engine, not the SM's load path).  Measured on the full
+            // event: 0.484 -> 0.395 ms per launch; issued after layer 1 (0.420) or layer 3 (0.412)
+            // it helps less.
+            const int nt = tile + 2 * (int)gridDim.x;
+            if (nt < p.n_tiles)
+              prefetch_l2_bulk(static_cast<const SE*>(p.e) + (size_t)nt * kTileRows * H, kTileRows * H * sizeof(SE));
+          }
           load_d(v);
           const float* vb = vecs + (2 + 3 * (l - 2)) * H;
           add_vec(v, vb);
@@ -889,6 +900,8 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           put_a(v);
           arrive_a(j, seq); next_job();                   // job: D = h * W_h^T
           GNN_TRACE_W(1);
+          if (KIND == TileKind::NodeUpdate && ws == 0 && lane == 0)   // this tile's aggregate rows
+            prefetch_l2_bulk(static_cast<const SE*>(p.agg) + (size_t)tile * kTileRows * H, kTileRows * H * sizeof(SE));
           // The aggregate rows are loaded only after the first job completed: a burst of global
           // loads from a slot's warps while its MMAs run slows those MMAs several-fold (the loads
           // compete with the tensor core's operand reads in the SM's memory pipeline).
@@ -912,6 +925,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         }
         if (l0 <= L) {                                    // last layer: new node state, and A for the P_s job
           wait_job();
+          if (KIND == TileKind::NodeUpdate && ws == 0 && lane == 0) {
+            // This slot's next h tile, ~10 us before its load.  Measured on the full event with the
+            // aggregate prefetch above: 0.223 -> 0.196 ms per launch; both tiles prefetched a whole
+            // tile ahead made it slower (0.248), prefetching later helps less.
+            const int nt = tile + 2 * (int)gridDim.x;
+            if (nt < p.n_tiles)
+              prefetch_l2_bulk(static_cast<const SE*>(p.h) + (size_t)nt * kTileRows * H, kTileRows * H * sizeof(SE));
+          }
           GNN_TRACE_W(3 + 2 * L);
           const float* vl = vb + 3 * (L - 1) * H;
           const bool w0 = ok && ok0, w1 = ok && ok1;
