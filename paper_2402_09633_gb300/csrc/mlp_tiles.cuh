@@ -164,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
   uint64_t* w_empty = bars + 4 + G::STAGES;          // [STAGES]  both slots' MMAs on a stage completed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * G::STAGES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  volatile int* progress = abort_flag + 1;          // [0] tile pair slot 0's workers are on (L2 prefetch pacing)
+  volatile int* progress = abort_flag + 1;          // [0] tile pair slot 0's workers are on (classifier L2 prefetch pacing)
                                                     // [1] slot 1 may start (edge kernels: the slots run out of phase)
 
   const int warp = threadIdx.x >> 5;
@@ -593,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 
       if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
         // vec layout: [gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]
-        if (slot == 0 && ws == 0 && lane == 0) progress[0] = pair;   // paces the L2 prefetcher
+        if (slot == 0 && ws == 0 && lane == 0) progress[0] = pair;   // paces the classifier's L2 prefetcher
         // The two slots run out of phase: slot 1 starts once slot 0 has released the last MMA of
         // its first tile, so that one slot's tile change (store, next loads) overlaps the other
         // slot's MMAs instead of leaving the tensor core idle.  Bounded: it starts anyway after
