@@ -153,7 +153,8 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
  * rounding per product and per sum, is below radius * radius (rounded to fp32) becomes one edge,
  * oriented from the hit with the smaller r (node_feats column 0; the smaller id on a tie).
  *   embedding  device float32 [n_nodes, emb_dim], emb_dim 1..16; unit vectors (as gnn_embed
- *              writes them) are searched on a grid over [-1, 1]^3, other values stay exact but
+ *              writes them) are searched on a grid over [-1, 1]^K (K = 4 for emb_dim >= 4,
+ *              else 3), other values stay exact but
  *              crowd into the grid's edge cells
  *   node_feats device float32 [n_nodes, n_node_feat] (column 0 orients the edges)
  *   edge_index device int32 with room for [2, max_edges], output: contiguous [2, n_edges]

@@ -3,17 +3,19 @@
 // nearest neighbours).
 //
 // The embeddings are unit vectors, so each coordinate lies in [-1, 1].  Hits
-// are binned on a uniform grid over their first three coordinates with cells
-// a little wider than half the radius (a coordinate outside [-1, 1] is clamped
-// to the edge cells, which keeps the search exact, only slower), and sorted by
-// cell (the library's stable radix sort); their embeddings and r values are
-// then gathered into that order, zero-padded to a multiple of four
-// coordinates.  A pair within the radius lies at most two cells apart on each
-// axis, so the partners of a hit sit in the 5 x 5 "rows" of cells around its
-// own, and in each row in one run of at most five consecutive cells, which is
-// one contiguous range of sorted positions.  Rows before the hit's own row hold
-// only earlier positions: each pair is visited once, by its earlier sorted
-// position, which scans 13 rows (its own row from the next position on).
+// are binned on a uniform grid over their first K coordinates (K = 4 when the
+// embedding has at least 4, else 3) with cells a little wider than half the
+// radius (a coordinate outside [-1, 1] is clamped to the edge cells, which
+// keeps the search exact, only slower), and sorted by cell (the library's
+// stable radix sort); their embeddings and r values are then gathered into
+// that order, zero-padded to a multiple of four coordinates.  A pair within
+// the radius lies at most two cells apart on each axis, so the partners of a
+// hit sit in the 5^(K-1) "rows" of cells around its own (rows over the first
+// K-1 gridded coordinates), and in each row in one run of at most five
+// consecutive cells along the last one, which is one contiguous range of
+// sorted positions.  Rows before the hit's own row hold only earlier positions:
+// each pair is visited once, by its earlier sorted position, which scans
+// (5^(K-1) + 1) / 2 rows (its own row from the next position on).
 //
 // The test is the full squared distance, summed over the coordinates in order
 // with one rounding per product and per sum (no fused multiply-add; the zero
@@ -28,14 +30,15 @@
 
 namespace gnn {
 
-constexpr int kFrnnMaxGrid = 128;        // cells per axis
 constexpr int kFrnnReach = 2;            // cells a partner can lie away on each axis
 
-// Cells per axis: cells 0.1 % wider than half the radius, so that the rounding of the cell
-// coordinates and of the distance test never puts a pair within the radius three cells apart.
-__host__ __device__ inline int frnn_grid(float radius) {
+// Cells per axis for a grid over K coordinates (K = 3 or 4): cells 0.1 % wider than half the radius,
+// so that the rounding of the cell coordinates and of the distance test never puts a pair within
+// the radius three cells apart; at most 128 (K = 3) or 64 (K = 4) cells per axis.
+__host__ __device__ inline int frnn_grid(float radius, int K) {
+  const int max_grid = K == 4 ? 64 : 128;
   const float cells = 1.998f * (float)kFrnnReach / radius;
-  return cells >= (float)kFrnnMaxGrid ? kFrnnMaxGrid : (cells < 1.0f ? 1 : (int)cells);
+  return cells >= (float)max_grid ? max_grid : (cells < 1.0f ? 1 : (int)cells);
 }
 
 __device__ __forceinline__ int frnn_coord(float e, int grid) {
@@ -43,15 +46,18 @@ __device__ __forceinline__ int frnn_coord(float e, int grid) {
   return c < 0 ? 0 : (c >= grid ? grid - 1 : c);
 }
 
+// Cell key of every hit: its cell over the first K coordinates (missing ones count as cell 0),
+// row-major with the last gridded coordinate fastest.
+template <int K>
 __global__ void frnn_cell_kernel(const float* __restrict__ emb, int n, int dim, int grid, int* __restrict__ keys,
                                  int* __restrict__ vals) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const float* e = emb + (size_t)i * dim;
-  const int c0 = frnn_coord(e[0], grid);
-  const int c1 = dim > 1 ? frnn_coord(e[1], grid) : 0;
-  const int c2 = dim > 2 ? frnn_coord(e[2], grid) : 0;
-  keys[i] = (c0 * grid + c1) * grid + c2;
+  int key = 0;
+#pragma unroll
+  for (int k = 0; k < K; ++k) key = key * grid + (k < dim ? frnn_coord(e[k], grid) : 0);
+  keys[i] = key;
   vals[i] = i;
 }
 
@@ -84,7 +90,36 @@ __device__ __forceinline__ float frnn_acc(float s, float a, float b) {
 // (Measured on the full event: separate counting and writing kernels, or a block-level scan of
 // the counts inside this kernel, made the search 12-22 % slower; the scan runs as separate
 // kernels between the passes instead.)
-template <int CH>
+// The candidate loop over one run of sorted positions [p, p1).
+#define GNN_FRNN_RUN()                                                                                   \
+  for (; p < p1; ++p) {                                                                                  \
+    float s = 0.f;                                                                                       \
+    _Pragma("unroll") for (int c = 0; c < CH; ++c) {                                                     \
+      const float4 e = emb_s[(size_t)p * CH + c];                                                        \
+      s = frnn_acc(s, q[c].x, e.x);                                                                      \
+      s = frnn_acc(s, q[c].y, e.y);                                                                      \
+      s = frnn_acc(s, q[c].z, e.z);                                                                      \
+      s = frnn_acc(s, q[c].w, e.w);                                                                      \
+    }                                                                                                    \
+    if (!(s < r2)) continue;                                                                             \
+    if (write) {                                                                                         \
+      const int j = ids[p];                                                                              \
+      const float rj = r_s[p];                                                                           \
+      const bool i_first = ri < rj || (ri == rj && i < j);                                               \
+      out[pos] = i_first ? i : j;                                                                        \
+      out[(size_t)n_total + pos] = i_first ? j : i;                                                      \
+      ++pos;                                                                                             \
+    } else {                                                                                             \
+      ++found;                                                                                           \
+    }                                                                                                    \
+  }
+
+// One thread per sorted position t.  write == 0: counts[t] = pairs visited from t;
+// write == 1: those pairs at offsets[t] (exclusive scan of counts), when the total fits.
+// (Measured on the full event: separate counting and writing kernels, or a block-level scan of
+// the counts inside this kernel, made the search 12-22 % slower; the scan runs as separate
+// kernels between the passes instead.)
+template <int CH, int K>
 __global__ void __launch_bounds__(256) frnn_pairs_kernel(
     const float4* __restrict__ emb_s, const float* __restrict__ r_s, int n, float r2, int grid,
     const int* __restrict__ cell_keys, const int* __restrict__ ids, const int* __restrict__ cell_start, int write,
@@ -104,49 +139,52 @@ __global__ void __launch_bounds__(256) frnn_pairs_kernel(
   float4 q[CH];
 #pragma unroll
   for (int c = 0; c < CH; ++c) q[c] = emb_s[(size_t)t * CH + c];
-  const int key = cell_keys[t];
-  const int c2 = key % grid, c1 = (key / grid) % grid, c0 = key / (grid * grid);
-  const int lo2 = c2 - kFrnnReach < 0 ? 0 : c2 - kFrnnReach;
-  const int hi2 = c2 + kFrnnReach >= grid ? grid - 1 : c2 + kFrnnReach;
+  int key = cell_keys[t];
+  const int cl = key % grid;                     // last gridded coordinate: the run axis
+  key /= grid;
+  const int lo = cl - kFrnnReach < 0 ? 0 : cl - kFrnnReach;
+  const int hi = cl + kFrnnReach >= grid ? grid - 1 : cl + kFrnnReach;
   int i = 0;
   float ri = 0.f;
   if (write) { i = ids[t]; ri = r_s[t]; }
   int found = 0;
-  for (int a = 0; a <= kFrnnReach; ++a) {
-    const int ra = c0 + a;
-    if (ra >= grid) break;
-    for (int b = (a == 0 ? 0 : -kFrnnReach); b <= kFrnnReach; ++b) {
-      const int rb = c1 + b;
-      if (rb < 0 || rb >= grid) continue;
-      const int row = (ra * grid + rb) * grid;
-      int p = cell_start[row + lo2];
-      const int p1 = cell_start[row + hi2 + 1];
-      if (a == 0 && b == 0) p = t + 1;
-      for (; p < p1; ++p) {
-        float s = 0.f;
-#pragma unroll
-        for (int c = 0; c < CH; ++c) {
-          const float4 e = emb_s[(size_t)p * CH + c];
-          s = frnn_acc(s, q[c].x, e.x);
-          s = frnn_acc(s, q[c].y, e.y);
-          s = frnn_acc(s, q[c].z, e.z);
-          s = frnn_acc(s, q[c].w, e.w);
-        }
-        if (!(s < r2)) continue;
-        if (write) {
-          const int j = ids[p];
-          const float rj = r_s[p];
-          const bool i_first = ri < rj || (ri == rj && i < j);
-          out[pos] = i_first ? i : j;
-          out[(size_t)n_total + pos] = i_first ? j : i;
-          ++pos;
-        } else {
-          ++found;
+  if constexpr (K == 3) {
+    const int c1 = key % grid, c0 = key / grid;
+    for (int a = 0; a <= kFrnnReach; ++a) {
+      const int ra = c0 + a;
+      if (ra >= grid) break;
+      for (int b = (a == 0 ? 0 : -kFrnnReach); b <= kFrnnReach; ++b) {
+        const int rb = c1 + b;
+        if (rb < 0 || rb >= grid) continue;
+        const int row = (ra * grid + rb) * grid;
+        int p = cell_start[row + lo];
+        const int p1 = cell_start[row + hi + 1];
+        if (a == 0 && b == 0) p = t + 1;
+        GNN_FRNN_RUN()
+      }
+    }
+  } else {
+    const int c2 = key % grid, c1 = (key / grid) % grid, c0 = key / (grid * grid);
+    for (int a = 0; a <= kFrnnReach; ++a) {
+      const int ra = c0 + a;
+      if (ra >= grid) break;
+      for (int b = (a == 0 ? 0 : -kFrnnReach); b <= kFrnnReach; ++b) {
+        const int rb = c1 + b;
+        if (rb < 0 || rb >= grid) continue;
+        for (int c = (a == 0 && b == 0 ? 0 : -kFrnnReach); c <= kFrnnReach; ++c) {
+          const int rc = c2 + c;
+          if (rc < 0 || rc >= grid) continue;
+          const int row = ((ra * grid + rb) * grid + rc) * grid;
+          int p = cell_start[row + lo];
+          const int p1 = cell_start[row + hi + 1];
+          if (a == 0 && b == 0 && c == 0) p = t + 1;
+          GNN_FRNN_RUN()
         }
       }
     }
   }
   if (!write) counts[t] = found;
 }
+#undef GNN_FRNN_RUN
 
 }  // namespace gnn

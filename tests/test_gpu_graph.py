@@ -78,6 +78,26 @@ def test_radius_graph_matches_oracle(n):
     net.close()
 
 
+@pytest.mark.parametrize("dim", [2, 5, 12])
+def test_radius_graph_other_embedding_widths(dim):
+    """D = 2 (grid over 3 coordinates, two of them real), 5 and 12 (grid over 4; one, two and three
+    float4 chunks per sorted embedding): edge sets bit-exact against the oracle."""
+    import torch
+    cfg = S.ModelConfig(12, 2, 64, 2, 2)
+    net, _, ew = _net(cfg, dim=dim)
+    x, _ = S.generate_event(S.EventSpec(4000, 9, "powerlaw", 0.02, n_edges=12000), 5)
+    xs = torch.from_numpy(x).cuda()
+    emb = net.embed(xs)
+    e_np = emb.cpu().numpy()
+    assert e_np.shape == (4000, dim)
+    np.testing.assert_allclose(e_np, O.embed(ew, x, cfg.ln_eps), atol=2e-4)
+    radius = _radius_for(e_np, 4)
+    ei, m = net.build_graph(emb, xs, radius, max_edges=200 * 4000)
+    assert m > 0
+    np.testing.assert_array_equal(_sorted_edges(ei.cpu().numpy()), _oracle_graph(e_np, x[:, 0], radius))
+    net.close()
+
+
 def test_radius_graph_full_event_sampled():
     """300k hits: the edges of 400 sampled hits against a brute-force search over every hit, and
     the properties every edge list must have (no self-loops, no duplicates, oriented by r)."""
