@@ -873,17 +873,19 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   const float r2 = radius * radius;
   const int xs = ctx->cfg.n_node_feat;
   const int sb = (N + kScanBlock - 1) / kScanBlock;
+  const int pb = (N + kFrnnPairsThreads - 1) / kFrnnPairsThreads;
   switch (chunks * 8 + K) {
 #define GNN_FRNN_CASE(CH, KK)                                                                                    \
   case CH * 8 + KK:                                                                                              \
     frnn_gather_kernel<CH><<<nb, tb, 0, st>>>(embedding, node_feats, xs, N, emb_dim, vin, emb_s, r_s);         \
-    frnn_pairs_kernel<CH, KK><<<nb, tb, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, 0, counts,      \
-                                                 nullptr, 0, nullptr, ctx->d_err);                              \
+    frnn_pairs_kernel<CH, KK><<<pb, kFrnnPairsThreads, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, \
+                                                                0, counts, nullptr, 0, nullptr, ctx->d_err);     \
     scan_reduce_kernel<<<sb, kScanBlock, 0, st>>>(counts, N, block_sums);                                      \
     compact_scan_kernel<<<1, 1024, 0, st>>>(block_sums, sb, n_edges);                                            \
     scan_apply_kernel<<<sb, kScanBlock, 0, st>>>(counts, N, block_sums);                                       \
-    frnn_pairs_kernel<CH, KK><<<nb, tb, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, 1, counts,      \
-                                                 n_edges, (int)max_edges, edge_index, ctx->d_err);              \
+    frnn_pairs_kernel<CH, KK><<<pb, kFrnnPairsThreads, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, \
+                                                                1, counts, n_edges, (int)max_edges, edge_index,  \
+                                                                ctx->d_err);                                     \
     break;
     GNN_FRNN_CASE(1, 3)
     GNN_FRNN_CASE(2, 3)
