@@ -231,6 +231,7 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           }
         }
       }
+      if (resident && lane == 0) drain_wait(&w_full[0], 0);     // the resident weights have landed
       if (!resident && lane == 0) {
         {
           uint32_t seq = 0;
@@ -243,6 +244,9 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
               bulk_g2s(ring + st * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[st]);
             }
           }
+          // before teardown, every copy this thread issued has landed (the last one per stage)
+          const uint32_t first = seq > (uint32_t)G::STAGES ? seq - G::STAGES : 0u;
+          for (uint32_t k = first; k < seq; ++k) drain_wait(&w_full[k % G::STAGES], (k / G::STAGES) & 1);
         }
       }
       __syncwarp();
@@ -317,6 +321,9 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
             }
           }
         }
+        // before teardown (and the TMEM release), this thread's last MMAs of each slot have completed
+        for (int s = 0; s < 2; ++s)
+          if (seq_s[s] > 0) drain_wait(&d_full[s], (seq_s[s] - 1) & 1);
       }
       __syncwarp();
     }

@@ -90,6 +90,17 @@ __device__ __forceinline__ bool bounded_wait(uint64_t* bar, uint32_t parity, vol
   }
 }
 
+// Teardown wait for this thread's own asynchronous work (a copy or an MMA commit) after the pipeline
+// may have aborted: ignores the abort flag, records nothing, and gives up after `limit_ns`.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns = 20000000ull) {
+  if (mbar_try_wait(bar, parity)) return;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait(bar, parity)) return;
+    if ((it & 63u) == 63u && global_timer_ns() - t0 > limit_ns) return;
+  }
+}
+
 // ------------------------------------------------------------- bulk copies
 // global -> shared, completion counted in bytes on `bar`.
 __device__ __forceinline__ void bulk_g2s(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
