@@ -241,12 +241,14 @@ int gnn_profile_read(gnn_ctx* ctx, double* ms, int64_t* launches, int n_groups);
 
 /*
  * gnn_status -- synchronise `stream`, then return and clear the device error
- * word of the context: GNN_OK, GNN_ERR_INDEX_RANGE, GNN_ERR_DEVICE_TIMEOUT or
- * GNN_ERR_CUDA (a failed synchronisation).
+ * word of the context: GNN_OK, GNN_ERR_INDEX_RANGE, GNN_ERR_DEVICE_TIMEOUT,
+ * GNN_ERR_CAPACITY (gnn_build_graph) or GNN_ERR_CUDA (a failed synchronisation).
  */
 int gnn_status(gnn_ctx* ctx, gnn_stream_t stream);
 
-/* gnn_destroy -- synchronise the device work of ctx and free it. NULL is a no-op. */
+/* gnn_destroy -- wait for the device (cudaDeviceSynchronize: the context does not know which
+ * streams used it, so other work on the device is waited for too) and free ctx and all its
+ * device memory. NULL is a no-op. */
 void gnn_destroy(gnn_ctx* ctx);
 
 /* gnn_error_string -- static text for a status code. */

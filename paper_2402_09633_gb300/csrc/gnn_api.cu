@@ -990,6 +990,9 @@ void gnn_destroy(gnn_ctx* ctx) {
   if (ctx->aux) cudaFree(ctx->aux);
   if (ctx->d_err) cudaFree(ctx->d_err);
   if (ctx->stage) cudaFree(ctx->stage);
+#ifdef GNN_TRACE
+  if (ctx->trace) cudaFree(ctx->trace);
+#endif
   for (auto& r : ctx->prof) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }
   delete ctx;
 }
