@@ -4,10 +4,15 @@
 One step = one gnn_infer call on one synthetic full event (300,000 nodes,
 1,000,000 candidate edges, 12 node features, H=128, T=8, 3-layer MLPs):
 device-side CSR build, encoders, eight message-passing iterations and the
-classifier, inputs resident in HBM.  Prints one JSON line (rank 0).  After the
-timed steps, `pipeline` times every stage of the tracking pipeline once more on
-the same event (embedding, graph building, filtering, the network, track
-labels); those stages are outside `value`.
+classifier, inputs resident in HBM.  Prints one JSON line (rank 0).  The
+headline steps are timed with nothing but their own CUDA events; the
+per-kernel split (`kernels`, and the dominant kernel's `roofline`) comes from a
+second pass with the library's profiling events between kernel groups.  After
+the timed steps, and outside `value`: `pipeline` times every stage of the
+tracking pipeline once on the same event (embedding, graph building,
+filtering, the network, track labels), `bf16` times the bf16 model on the same
+event and `batch16` one call on 16 events (4.8M nodes, 16M edges), each with
+its own step roofline.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
 
@@ -289,6 +294,92 @@ def run_pipeline(net, w: S.Workload, x, dev, reps: int = 5):
     return out
 
 
+def time_steps(net, x, ei, scores, flush, stream, steps: int):
+    """Device time (ms) of `steps` gnn_infer calls, one CUDA event pair per call on the launching
+    stream, with the L2 flushed (a buffer of twice its size written) before each call."""
+    import torch
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    for k in range(steps):
+        flush.fill_(float(k))
+        starts[k].record(stream)
+        net.infer(x, ei, scores)
+        ends[k].record(stream)
+    torch.cuda.synchronize()
+    return [a.elapsed_time(b) for a, b in zip(starts, ends)]
+
+
+def kernel_split(net, x, ei, scores, flush, stream, steps: int):
+    """Per-kernel-group device time from a separate pass of `steps` calls with the library's
+    profiling events on (they sit between kernel groups, so the headline is timed without them)."""
+    net.profile(True)
+    net.profile_read()                                   # clear
+    ms = time_steps(net, x, ei, scores, flush, stream, steps)
+    prof = net.profile_read()
+    net.profile(False)
+    groups = {g: {"ms_total": t, "launches": n, "ms_per_launch": t / n} for g, (t, n) in prof.items() if n}
+    return groups, sum(ms) / len(ms)
+
+
+def cpu_model() -> str:
+    """Host CPU model name, from lscpu or /proc/cpuinfo."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu model")):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.machine()
+
+
+def side_workload(name: str, steps: int, dev, peaks, x_dev=None, ei_dev=None):
+    """One more workload timed after the headline (outside its timed region): the bf16 model on the
+    same event, or the 16-event batch in one call.  Returns its sub-object of the JSON line."""
+    import torch
+    from paper_2402_09633_gb300 import InteractionNetwork
+    w = S.WORKLOADS[name]
+    if x_dev is None:
+        x_np, ei_np = (S.generate_batch(w.event, list(w.seeds)) if w.n_events > 1
+                       else S.generate_event(w.event, w.seeds[0]))
+        x_dev, ei_dev = torch.from_numpy(x_np).to(dev), torch.from_numpy(ei_np).to(dev)
+    N, E = x_dev.shape[0], ei_dev.shape[1]
+    net = InteractionNetwork(w.model, S.pack_blob(w.model, S.init_weights(w.model, w.weight_seed)))
+    net.reserve(N, E)
+    scores = torch.empty(E, dtype=torch.float32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    time_steps(net, x_dev, ei_dev, scores, flush, stream, 3)
+    ms = time_steps(net, x_dev, ei_dev, scores, flush, stream, steps)
+    status = net.status()
+    groups, _ = kernel_split(net, x_dev, ei_dev, scores, flush, stream, min(steps, 5))
+    net.close()
+    mean_ms = sum(ms) / len(ms)
+    model = step_model(w)
+    t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9), model["flops"] / (peaks["bf16_tflops"] * 1e12))
+    out = {"workload": name, "description": w.description, "n_nodes": N, "n_edges": E,
+           "steps": steps, "ms_per_step": mean_ms, "edges_per_s": E / (mean_ms * 1e-3),
+           "events_per_s": w.n_events / (mean_ms * 1e-3),
+           "dtype": "bf16->f32" if w.model.precision == S.PRECISION_BF16 else "bf16x3->f32",
+           "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms, "bytes_alg": model["bytes"],
+                             "flops_alg": model["flops"], "bytes_per_activation": 2 if w.model.precision else 4},
+           "kernels": {g: v["ms_per_launch"] for g, v in groups.items()}, "device_status": status}
+    if w.model.precision == S.PRECISION_BF16:
+        out["tolerance"] = ("stated 1e-2 max on logits is not met: the GPU's max logit error against the "
+                            "fp64 oracle exceeds it on the full event, as does the oracle's own fp64-vs-fp32 "
+                            "evaluation of the same bf16 model; tests/test_gpu_bf16.py checks the error's "
+                            "distribution against that envelope")
+    return out
+
+
 def run_gb300(args, rank: int, world: int, local: int):
     import torch
     import torch.distributed as dist
@@ -316,40 +407,30 @@ def run_gb300(args, rank: int, world: int, local: int):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    for _ in range(args.warmup):
-        flush.fill_(1.0)
-        net.infer(x, ei, scores)
-    torch.cuda.synchronize(dev)
+    time_steps(net, x, ei, scores, flush, stream, args.warmup)
     if net.status() != 0:
         raise RuntimeError("device error during warm-up")
 
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    # headline: exactly `steps` timed calls, no profiling events inside
     sampler = ClockSampler(gpu_index_for(local))
     time.sleep(0.3)
-    net.profile(True)
-    net.profile_read()                                   # clear
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
     t_wall = time.perf_counter()
-    for k in range(args.steps):
-        flush.fill_(float(k))
-        starts[k].record(stream)
-        net.infer(x, ei, scores)
-        ends[k].record(stream)
-    torch.cuda.synchronize(dev)
+    step_ms = time_steps(net, x, ei, scores, flush, stream, args.steps)
     if world > 1:
         dist.barrier()
     wall = time.perf_counter() - t_wall
     clocks = sampler.stop()
-    prof = net.profile_read()
-    net.profile(False)
     status = net.status()
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     step_s, job_edges = whole_job(sum(step_ms) / len(step_ms) * 1e-3, E, world, dev)
     mean_ms = step_s * 1e3
     value = job_edges / step_s
+
+    # per-kernel split: a second pass with the library's profiling events
+    split_steps = max(3, min(args.steps, 20))
+    groups, profiled_ms = kernel_split(net, x, ei, scores, flush, stream, split_steps)
 
     # end to end through the host-buffer entry point (copies inside the timed region)
     x_h = torch.from_numpy(x_np).pin_memory()
@@ -370,33 +451,44 @@ def run_gb300(args, rank: int, world: int, local: int):
             dist.destroy_process_group()
         return
 
-    pipeline = run_pipeline(net, w, x, dev) if w.n_events == 1 else None
-
     peaks, peak_src = load_peaks()
+    side = {}
+    if world == 1 and not args.no_side_workloads and args.workload == "full":
+        pipeline = run_pipeline(net, w, x, dev)
+        net.close()
+        side["bf16"] = side_workload("full_bf16", max(3, min(args.steps, 50)), dev, peaks, x, ei)
+        side["batch16"] = side_workload("batch16", max(3, min(args.steps, 10)), dev, peaks)
+    else:
+        pipeline = run_pipeline(net, w, x, dev) if w.n_events == 1 else None
+        net.close()
+
     model = step_model(w)
-    groups = {g: {"ms_total": ms, "launches": n} for g, (ms, n) in prof.items() if n}
     kernels_only = {g: v for g, v in groups.items() if g != "host_copies"}
     dom = max(kernels_only, key=lambda g: kernels_only[g]["ms_total"])
-    dom_avg_s = kernels_only[dom]["ms_total"] * 1e-3 / kernels_only[dom]["launches"]
+    dom_avg_s = kernels_only[dom]["ms_per_launch"] * 1e-3
     dom_model = model.get(dom, None)
     roofline = None
     if dom_model is not None:
         achieved = dom_model["bytes"] / dom_avg_s / 1e9
         roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"],
-                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": profiled_traffic(dom, w.model.precision == S.PRECISION_BF16),
+                    "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                    "traffic": profiled_traffic(dom, w.model.precision == S.PRECISION_BF16),
                     "peak_source": f"{peak_src} (hbm_gbs, copy burst) -- of {peak_src}",
                     "bytes_per_launch": dom_model["bytes"], "avg_launch_ms": dom_avg_s * 1e3,
+                    "launch_timing": f"CUDA events around each launch on the launching stream, "
+                                     f"{split_steps} profiled steps after the headline",
                     "tensor_tflops_executed": (1 if w.model.precision == S.PRECISION_BF16 else 3)
                                               * dom_model["flops"] / dom_avg_s / 1e12}
     t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9),
                           model["flops"] / (peaks["bf16_tflops"] * 1e12))
-    total_launches = sum(v["launches"] for v in kernels_only.values())
+    launches_per_step = sum(v["launches"] for v in kernels_only.values()) / split_steps
 
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         scale = 0.1
         e_s, n_s, t = time_oracle(w, scale, 1)
         cpu = {"value": e_s / t[0], "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "cpu_model": cpu_model(), "threads": cpu_cores(),
                "sample": f"{n_s} nodes / {e_s} edges from the '{w.name}' generator ({scale:g} of the "
                          f"event), same model, fp64 numpy, one pass of {t[0]:.1f} s"}
 
@@ -410,13 +502,15 @@ def run_gb300(args, rank: int, world: int, local: int):
             "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms,
                               "bytes_alg": model["bytes"], "flops_alg": model["flops"]},
             "kernels": groups,
+            "kernels_pass": {"steps": split_steps, "ms_per_step_with_events": profiled_ms},
+            **side,
             "pipeline": pipeline,
             "cpu_baseline": cpu,
             "e2e": {"value": job_edges / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": int(x_np.nbytes + ei_np.nbytes),
                     "d2h_bytes_per_step": int(E * 4), "ms_per_step": e2e_s * 1e3,
                     "matches_device_path": e2e_ok},
-            "gpu_launches": int(total_launches),
+            "gpu_launches": int(round(launches_per_step * args.steps)),
             "clocks": clocks,
             "device_status": status,
             "wall_s_timed_region": wall}
@@ -433,6 +527,8 @@ def main():
     ap.add_argument("--impl", choices=("gb300", "reference"), default="gb300")
     ap.add_argument("--workload", choices=tuple(S.WORKLOADS), default="full")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-side-workloads", action="store_true",
+                    help="skip the bf16-model and 16-event-batch sub-objects (timed after the headline)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
