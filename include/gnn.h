@@ -40,6 +40,11 @@ extern "C" {
 
 typedef struct CUstream_st* gnn_stream_t; /* a cudaStream_t; NULL = legacy default stream */
 
+/* The largest count any call accepts (nodes, edges, an output capacity): 2^31 - 1 - 8192, so that
+ * the kernels' 32-bit row indices stay in range after rounding up to whole blocks and tiles.  A
+ * larger count (or a negative one) is INVALID_ARG, returned before any device work. */
+#define GNN_MAX_COUNT 2147475455
+
 enum gnn_status_code {
   GNN_OK = 0,
   GNN_ERR_INVALID_ARG = -1,    /* null pointer, bad size or unsupported configuration */
@@ -109,7 +114,7 @@ int gnn_reserve(gnn_ctx* ctx, int64_t max_nodes, int64_t max_edges);
  *
  * All three buffers are caller-owned and must stay valid until the stream
  * reaches this work; the library never frees them.  n_edges == 0 is a no-op;
- * n_nodes == 0 with n_edges > 0 and sizes above INT32_MAX - 1 are
+ * n_nodes == 0 with n_edges > 0 and sizes above GNN_MAX_COUNT are
  * INVALID_ARG.  The workspace grows here (synchronous allocation) when the
  * graph is larger than any earlier one; call gnn_reserve first to avoid it.
  * An edge with an endpoint outside [0, n_nodes) gets a NaN score, takes no
@@ -216,9 +221,10 @@ int gnn_filter_edges(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_
  *
  * Edges with an endpoint outside [0, n_nodes) are skipped.  The labels do not depend on thread
  * or edge order.  Enqueued on `stream`; uses no workspace (the labels array is the union-find
- * forest).  A union retry loop that never settles records GNN_ERR_DEVICE_TIMEOUT in the context's
- * device error word (see gnn_status).  Errors: INVALID_ARG (null pointer, negative or too large
- * sizes, n_nodes == 0 with edges), CUDA.
+ * forest).  Every union and find loop gives up after 1 s of wall-clock time (%globaltimer) and
+ * then records GNN_ERR_DEVICE_TIMEOUT in the context's device error word (see gnn_status); the
+ * labels are then invalid.  Errors: INVALID_ARG (null pointer, negative sizes or sizes above
+ * GNN_MAX_COUNT, n_nodes == 0 with edges), CUDA.
  */
 int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge_index, int64_t n_nodes,
                      int64_t n_edges, float threshold, int32_t* labels, gnn_stream_t stream);
@@ -301,13 +307,17 @@ int gnn_debug_wait_timeout(gnn_ctx* ctx, int64_t limit_ns, gnn_stream_t stream);
  *   src_sorted device int32 [n_edges]: source of each sorted slot
  * The result is bit-identical to the CSR gnn_infer builds: edges stably
  * sorted by destination (ties keep input order).  Edges with an endpoint
- * outside [0, n_nodes) are placed after rowptr[n_nodes] (so rowptr[n_nodes]
- * < n_edges reveals them) with source 0.
- * Limits: n_edges <= GNN_CSR_NOALLOC_MAX_EDGES and 0 <= n_nodes < INT32_MAX;
+ * outside [0, n_nodes) are placed after rowptr[n_nodes], in input order,
+ * with source 0: rowptr[n_nodes] < n_edges is the only signal of them (this
+ * call has no context, so no error word records them).
+ * Limits: n_edges <= GNN_CSR_NOALLOC_MAX_EDGES and 0 <= n_nodes <= GNN_MAX_COUNT;
  * larger sizes, negative sizes or null pointers return GNN_ERR_INVALID_ARG
- * before any device work.  The first call on a device looks up the scratch
- * array's device address (device set-up; make that first call outside any
- * stream capture).  All calls share the one array and it keeps the last
+ * before any device work.  Every call looks up the scratch array's device
+ * address in the current context (cudaGetSymbolAddress: it allocates and
+ * enqueues nothing, and follows the array when a device reset or another
+ * context gives it a new address); the first call in a context may load the
+ * library's device code, so make that first call outside any stream capture.
+ * All calls share the one array and it keeps the last
  * call's contents (nothing in it needs to start at zero); calls that overlap
  * on the GPU (several streams, or several host threads) race on it and must
  * be serialised by the caller.  Enqueued on `stream`; no host synchronisation.

@@ -20,10 +20,12 @@ constexpr int kRadixThreads = 256;
 constexpr int kRadixRounds = 16;
 constexpr int kRadixTile = kRadixThreads * kRadixRounds;   // elements per tile
 
-// K0: endpoint validation and sort keys.
+// K0: endpoint validation and sort keys.  An out-of-range edge sets DEV_ERR_INDEX_RANGE in *err
+// (when err is not null) and sorts last (key n_nodes).
 __global__ void csr_keys_kernel(const int32_t* __restrict__ ei, int n_edges, int n_nodes,
                                 int* __restrict__ keys, int* __restrict__ vals,
                                 int* __restrict__ src_clamped, uint32_t* err) {
+  pdl_wait();
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= n_edges) return;
   const int s = ei[k];
@@ -32,12 +34,13 @@ __global__ void csr_keys_kernel(const int32_t* __restrict__ ei, int n_edges, int
   keys[k] = ok ? d : n_nodes;
   vals[k] = k;
   src_clamped[k] = ok ? s : 0;
-  if (!ok) atomicOr(err, DEV_ERR_INDEX_RANGE);
+  if (!ok && err) atomicOr(err, DEV_ERR_INDEX_RANGE);
 }
 
 // Per-tile digit histogram: hist[tile * 256 + digit].
 __global__ void radix_count_kernel(const int* __restrict__ keys, int n, int shift, int n_tiles,
                                    int* __restrict__ hist) {
+  pdl_wait();
   __shared__ int cnt[256];
   cnt[threadIdx.x] = 0;
   __syncthreads();
@@ -55,6 +58,7 @@ __global__ void radix_count_kernel(const int* __restrict__ keys, int n, int shif
 // earlier tiles.  One block of 256 threads; thread d walks its digit's column
 // (reads are coalesced across threads), then the 256 digit totals are scanned.
 __global__ void __launch_bounds__(256) radix_offsets_kernel(int* __restrict__ hist, int n_tiles) {
+  pdl_wait();
   __shared__ int tot[256];
   const int d = threadIdx.x;
   int run = 0;
@@ -82,6 +86,7 @@ __global__ void __launch_bounds__(256) radix_offsets_kernel(int* __restrict__ hi
 __global__ void radix_scatter_kernel(const int* __restrict__ keys_in, const int* __restrict__ vals_in,
                                      int* __restrict__ keys_out, int* __restrict__ vals_out, int n,
                                      int shift, int n_tiles, const int* __restrict__ offs) {
+  pdl_wait();
   __shared__ int run[256];
   __shared__ int wcnt[kRadixThreads / 32][256];
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
@@ -121,6 +126,7 @@ __global__ void csr_gather_kernel(const int* __restrict__ keys_sorted, const int
                                   const int* __restrict__ src_clamped, int n_edges, int n_nodes,
                                   int* __restrict__ perm, int* __restrict__ src_sorted,
                                   int* __restrict__ dst_sorted) {
+  pdl_wait();
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= n_edges) return;
   const int id = vals_sorted[k];
@@ -133,6 +139,7 @@ __global__ void csr_gather_kernel(const int* __restrict__ keys_sorted, const int
 // rowptr[j] = first sorted slot whose key >= j (binary search), for j in [0, n_nodes].
 __global__ void csr_rowptr_kernel(const int* __restrict__ keys_sorted, int n_edges, int n_nodes,
                                   int* __restrict__ rowptr) {
+  pdl_wait();
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j > n_nodes) return;
   int lo = 0, hi = n_edges;

@@ -19,8 +19,8 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
-#include <mutex>
 #include <new>
+#include <utility>
 #include <vector>
 
 #include "../../include/gnn.h"
@@ -206,6 +206,34 @@ int cuda_fail(cudaError_t e) {
   return e == cudaErrorMemoryAllocation ? GNN_ERR_OOM : GNN_ERR_CUDA;
 }
 
+// Every count a call accepts (nodes, edges, output capacity) lies in [0, GNN_MAX_COUNT], so that
+// the kernels' 32-bit row indices stay in range after rounding up to a whole block or radix tile
+// (at most 8192 rows).
+inline bool count_ok(int64_t n) { return n >= 0 && n <= (int64_t)GNN_MAX_COUNT; }
+
+// Blocks of `per_block` threads (or rows) covering n, computed in 64 bits.
+inline unsigned blocks_for(int64_t n, int64_t per_block) { return (unsigned)((n + per_block - 1) / per_block); }
+
+// Launch as a programmatic dependent of the previous kernel in the stream: the kernel may start
+// while that one finishes its last CTAs, and waits for it (pdl_wait) before touching its data.
+// Every kernel launched this way calls pdl_wait before its first access to data an earlier
+// kernel writes.  Returns the launch status.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 constexpr int kProfGroups = 10;
 
 // Returns the record index, or -1 when profiling is off.
@@ -245,7 +273,7 @@ cudaError_t set_all_attrs() {
 }
 
 template <TileKind K, int H, bool BF>
-void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st) {
+cudaError_t launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st) {
   p.n_jobs = pl.n_jobs;
   for (int j = 0; j < kMaxJobs; ++j) { p.job_mat[j] = pl.job_mat[j]; p.job_acc[j] = pl.job_acc[j]; }
   p.vecs = pl.d_vecs;
@@ -253,7 +281,7 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
   p.wmats = pl.wmats ? pl.wmats : c->d_mats;
   p.mat_bytes = c->mat_bytes;
   p.n_tiles = (p.n_rows + kTileRows - 1) / kTileRows;
-  if (p.n_tiles == 0) return;
+  if (p.n_tiles == 0) return cudaSuccess;
   const uint32_t smem = tile_launch_smem<H, BF>(p.n_vec_floats);
   const int grid = tile_grid(p.n_tiles, c->n_sm);
 #ifdef GNN_TRACE
@@ -261,8 +289,9 @@ void launch_tile(gnn_ctx* c, const KernelPlan& pl, TileParams p, cudaStream_t st
 #endif
   static const int group[7] = {1, 2, 3, 4, 5, 8, 9};   // NodeEncoder, EdgeEncoder, EdgeUpdate, NodeUpdate, Classifier, Filter, Embed
   const int pr = prof_begin(c, group[(int)K], 1, st);
-  mlp_tile_kernel<K, H, BF><<<grid, kThreads, smem, st>>>(p);
+  const cudaError_t err = launch_pdl(mlp_tile_kernel<K, H, BF>, grid, kThreads, smem, st, p);
   prof_end(c, pr, st);
+  return err;
 }
 
 template <int H, bool BF>
@@ -283,22 +312,24 @@ int run_network(gnn_ctx* c, const float* x, int N, int E, float* scores, cudaStr
   p.err = c->d_err;
   const int T = c->cfg.n_iters;
 
+  cudaError_t le = cudaSuccess;                        // first launch error
+  auto chk = [&](cudaError_t e) { if (le == cudaSuccess) le = e; };
   TileParams pn = p; pn.n_rows = N; pn.n_feat = c->cfg.n_node_feat;
-  launch_tile<TileKind::NodeEncoder, H, BF>(c, c->plan[T > 0 ? 0 : 1], pn, st);
+  chk(launch_tile<TileKind::NodeEncoder, H, BF>(c, c->plan[T > 0 ? 0 : 1], pn, st));
   TileParams pe = p; pe.n_rows = E; pe.n_feat = 2;
-  launch_tile<TileKind::EdgeEncoder, H, BF>(c, c->plan[2], pe, st);
+  chk(launch_tile<TileKind::EdgeEncoder, H, BF>(c, c->plan[2], pe, st));
   for (int t = 1; t <= T; ++t) {
-    launch_tile<TileKind::EdgeUpdate, H, BF>(c, c->plan[3], pe, st);
+    chk(launch_tile<TileKind::EdgeUpdate, H, BF>(c, c->plan[3], pe, st));
     {
       const int pr = prof_begin(c, 7, 1, st);
-      constexpr int npb = agg_nodes_per_block<H>();
-      aggregate_kernel<H, BF><<<(N + npb - 1) / npb, 256, 0, st>>>(c->e, c->rowptr, N, c->agg);
+      chk(launch_pdl(aggregate_kernel<H, BF>, blocks_for(N, agg_nodes_per_block<H>()), 256, 0, st, (const void*)c->e,
+                     (const int*)c->rowptr, N, c->agg));
       prof_end(c, pr, st);
     }
-    launch_tile<TileKind::NodeUpdate, H, BF>(c, c->plan[t < T ? 4 : 5], pn, st);
+    chk(launch_tile<TileKind::NodeUpdate, H, BF>(c, c->plan[t < T ? 4 : 5], pn, st));
   }
-  launch_tile<TileKind::Classifier, H, BF>(c, c->plan[6], pe, st);
-  const cudaError_t err = cudaGetLastError();
+  chk(launch_tile<TileKind::Classifier, H, BF>(c, c->plan[6], pe, st));
+  const cudaError_t err = le != cudaSuccess ? le : cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
 
@@ -353,27 +384,30 @@ int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
   while (n_bits < 31 && (N >> n_bits) != 0) ++n_bits;
   const int n_passes = ((n_bits > 0 ? n_bits : 1) + 7) / 8;
   const int pr = prof_begin(c, 0, 3 + 3 * n_passes, st);
-  csr_keys_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(ei, E, N, c->keys_a, c->vals_a, c->src_c, c->d_err);
+  cudaError_t le = cudaSuccess;                        // first launch error
+  auto chk = [&](cudaError_t e) { if (le == cudaSuccess) le = e; };
+  chk(launch_pdl(csr_keys_kernel, blocks_for(E, tb), tb, 0, st, ei, E, N, c->keys_a, c->vals_a, c->src_c, c->d_err));
   int bits = 0;
   while (bits < 31 && (N >> bits) != 0) ++bits;        // keys lie in [0, N]
   if (bits == 0) bits = 1;
   const int passes = (bits + 7) / 8;
-  const int tiles = (E + kRadixTile - 1) / kRadixTile;
+  const int tiles = (int)blocks_for(E, kRadixTile);
   int *kin = c->keys_a, *vin = c->vals_a, *kout = c->keys_b, *vout = c->vals_b;
   for (int ps = 0; ps < passes; ++ps) {
     const int shift = 8 * ps;
-    radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, E, shift, tiles, c->hist);
-    radix_offsets_kernel<<<1, 256, 0, st>>>(c->hist, tiles);
-    radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, E, shift, tiles, c->hist);
+    chk(launch_pdl(radix_count_kernel, tiles, kRadixThreads, 0, st, (const int*)kin, E, shift, tiles, c->hist));
+    chk(launch_pdl(radix_offsets_kernel, 1, 256, 0, st, c->hist, tiles));
+    chk(launch_pdl(radix_scatter_kernel, tiles, kRadixThreads, 0, st, (const int*)kin, (const int*)vin, kout, vout, E,
+                   shift, tiles, (const int*)c->hist));
     int* t = kin; kin = kout; kout = t;
     t = vin; vin = vout; vout = t;
   }
   c->key_sorted = kin;
-  csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, c->src_c, E, N, c->perm, c->src_sorted,
-                                                     c->dst_sorted);
-  csr_rowptr_kernel<<<(N + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, c->rowptr);
+  chk(launch_pdl(csr_gather_kernel, blocks_for(E, tb), tb, 0, st, (const int*)kin, (const int*)vin,
+                 (const int*)c->src_c, E, N, c->perm, c->src_sorted, c->dst_sorted));
+  chk(launch_pdl(csr_rowptr_kernel, blocks_for((int64_t)N + 1, tb), tb, 0, st, (const int*)kin, E, N, c->rowptr));
   prof_end(c, pr, st);
-  const cudaError_t err = cudaGetLastError();
+  const cudaError_t err = le != cudaSuccess ? le : cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
 
@@ -558,15 +592,13 @@ int gnn_create(const gnn_config* cfg, const void* weights_host, size_t weights_b
 }
 
 int gnn_reserve(gnn_ctx* ctx, int64_t max_nodes, int64_t max_edges) {
-  if (!ctx || max_nodes < 0 || max_edges < 0 || max_nodes >= INT32_MAX || max_edges >= INT32_MAX)
-    return GNN_ERR_INVALID_ARG;
+  if (!count_ok(max_nodes) || !count_ok(max_edges) || !ctx) return GNN_ERR_INVALID_ARG;
   return ensure_workspace(ctx, max_nodes, max_edges);
 }
 
 int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
               int64_t n_edges, float* edge_scores, gnn_stream_t stream) {
-  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX)
-    return GNN_ERR_INVALID_ARG;
+  if (!count_ok(n_nodes) || !count_ok(n_edges) || !ctx) return GNN_ERR_INVALID_ARG;
   if (n_edges == 0) return GNN_OK;
   if (n_nodes == 0 || !node_feats || !edge_index || !edge_scores) return GNN_ERR_INVALID_ARG;
   int rc = ensure_workspace(ctx, n_nodes, n_edges);
@@ -587,8 +619,7 @@ int gnn_infer(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, 
 
 int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
                    int64_t n_edges, float* edge_scores, gnn_stream_t stream) {
-  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX)
-    return GNN_ERR_INVALID_ARG;
+  if (!count_ok(n_nodes) || !count_ok(n_edges) || !ctx) return GNN_ERR_INVALID_ARG;
   if (n_edges == 0) return GNN_OK;
   if (n_nodes == 0 || !node_feats || !edge_index || !edge_scores) return GNN_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;
@@ -685,8 +716,7 @@ int gnn_filter_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes
 int gnn_filter_edges(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_index, int64_t n_nodes,
                      int64_t n_edges, float threshold, float* edge_scores, int32_t* kept_index, int32_t* kept_id,
                      int32_t* n_kept, gnn_stream_t stream) {
-  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX || !n_kept)
-    return GNN_ERR_INVALID_ARG;
+  if (!count_ok(n_nodes) || !count_ok(n_edges) || !ctx || !n_kept) return GNN_ERR_INVALID_ARG;
   if (ctx->filter_layers == 0) return GNN_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;
   if (n_edges == 0) {
@@ -716,7 +746,7 @@ int gnn_filter_edges(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_
     if (bf) launch_tile<TileKind::Filter, 64, true>(ctx, ctx->filter_plan, p, st);
     else launch_tile<TileKind::Filter, 64, false>(ctx, ctx->filter_plan, p, st);
   }
-  const int nb = (E + kCompactBlock - 1) / kCompactBlock;
+  const int nb = (int)blocks_for(E, kCompactBlock);
   int* counts = ctx->keys_a;
   compact_count_kernel<<<nb, kCompactThreads, 0, st>>>(edge_scores, E, threshold, counts);
   compact_scan_kernel<<<1, 1024, 0, st>>>(counts, nb, n_kept);
@@ -789,7 +819,7 @@ int gnn_embed_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes)
 }
 
 int gnn_embed(gnn_ctx* ctx, const float* node_feats, int64_t n_nodes, float* embedding, gnn_stream_t stream) {
-  if (!ctx || n_nodes < 0 || n_nodes >= INT32_MAX || ctx->embed_layers == 0) return GNN_ERR_INVALID_ARG;
+  if (!count_ok(n_nodes) || !ctx || ctx->embed_layers == 0) return GNN_ERR_INVALID_ARG;
   if (n_nodes == 0) return GNN_OK;
   if (!node_feats || !embedding) return GNN_ERR_INVALID_ARG;
   TileParams p{};
@@ -818,8 +848,8 @@ int gnn_embed(gnn_ctx* ctx, const float* node_feats, int64_t n_nodes, float* emb
 
 int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const float* node_feats, int64_t n_nodes,
                     float radius, int64_t max_edges, int32_t* edge_index, int32_t* n_edges, gnn_stream_t stream) {
-  if (!ctx || n_nodes < 0 || n_nodes >= INT32_MAX || emb_dim < 1 || emb_dim > kMaxEmbedDim || !(radius > 0.f) ||
-      max_edges < 0 || max_edges >= INT32_MAX || !n_edges)
+  if (!count_ok(n_nodes) || !count_ok(max_edges) || !ctx || emb_dim < 1 || emb_dim > kMaxEmbedDim ||
+      !(radius > 0.f) || !n_edges)
     return GNN_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;
   if (n_nodes == 0) {
@@ -834,11 +864,11 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   const int grid = frnn_grid(radius, K);
   int n_cells = 1;
   for (int k = 0; k < K; ++k) n_cells *= grid;
-  const int tiles = (N + kRadixTile - 1) / kRadixTile;
+  const int tiles = (int)blocks_for(N, kRadixTile);
   const int chunks = (emb_dim + 3) / 4;                   // float4 chunks per sorted embedding
   // scratch: emb_s [N, 4 * chunks] (first, 16-byte aligned), r_s, keys/vals (two buffers each),
   // per-hit counts, per-block sums, radix histograms, cell starts
-  const int nb = (N + tb - 1) / tb;
+  const int nb = (int)blocks_for(N, tb);
   const size_t need = 4 * (size_t)chunks * N + 6 * (size_t)N + (size_t)nb + 256 * (size_t)tiles + (size_t)n_cells + 1;
   if (need > ctx->aux_ints) {
     if (ctx->aux) { cudaStreamSynchronize(st); cudaFree(ctx->aux); ctx->aux = nullptr; ctx->aux_ints = 0; }
@@ -869,11 +899,11 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
     int* t = kin; kin = kout; kout = t;
     t = vin; vin = vout; vout = t;
   }
-  csr_rowptr_kernel<<<(n_cells + 1 + tb - 1) / tb, tb, 0, st>>>(kin, N, n_cells, cell_start);
+  csr_rowptr_kernel<<<blocks_for((int64_t)n_cells + 1, tb), tb, 0, st>>>(kin, N, n_cells, cell_start);
   const float r2 = radius * radius;
   const int xs = ctx->cfg.n_node_feat;
-  const int sb = (N + kScanBlock - 1) / kScanBlock;
-  const int pb = (N + kFrnnPairsThreads - 1) / kFrnnPairsThreads;
+  const int sb = (int)blocks_for(N, kScanBlock);
+  const int pb = (int)blocks_for(N, kFrnnPairsThreads);
   switch (chunks * 8 + K) {
 #define GNN_FRNN_CASE(CH, KK)                                                                                    \
   case CH * 8 + KK:                                                                                              \
@@ -903,15 +933,15 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
 
 int gnn_track_labels(gnn_ctx* ctx, const float* edge_scores, const int32_t* edge_index, int64_t n_nodes,
                      int64_t n_edges, float threshold, int32_t* labels, gnn_stream_t stream) {
-  if (!ctx || n_nodes < 0 || n_edges < 0 || n_nodes >= INT32_MAX || n_edges >= INT32_MAX) return GNN_ERR_INVALID_ARG;
+  if (!count_ok(n_nodes) || !count_ok(n_edges) || !ctx) return GNN_ERR_INVALID_ARG;
   if (n_nodes == 0) return n_edges == 0 ? GNN_OK : GNN_ERR_INVALID_ARG;
   if (!labels || (n_edges > 0 && (!edge_scores || !edge_index))) return GNN_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;
   const int N = (int)n_nodes, E = (int)n_edges, tb = 256;
-  cc_init_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
-  if (E > 0) cc_union_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(edge_scores, edge_index, N, E, threshold, labels, ctx->d_err);
-  cc_compress_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
-  cc_flatten_kernel<<<(N + tb - 1) / tb, tb, 0, st>>>(labels, N);
+  cc_init_kernel<<<blocks_for(N, tb), tb, 0, st>>>(labels, N);
+  if (E > 0) cc_union_kernel<<<blocks_for(E, tb), tb, 0, st>>>(edge_scores, edge_index, N, E, threshold, labels, ctx->d_err);
+  cc_compress_kernel<<<blocks_for(N, tb), tb, 0, st>>>(labels, N, ctx->d_err);
+  cc_flatten_kernel<<<blocks_for(N, tb), tb, 0, st>>>(labels, N, ctx->d_err);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? GNN_OK : cuda_fail(err);
 }
@@ -1022,55 +1052,27 @@ int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_
 // device array instead of context workspace.  Layout (int32 words):
 // keys_a | keys_b | vals_a | vals_b | src_clamped (GNN_CSR_NOALLOC_MAX_EDGES
 // each) | per-tile digit histograms (256 x 256).  Host code must not use the
-// array's name as a device address: the address comes from
-// cudaGetSymbolAddress, looked up once per device with that device current.
+// array's name as a device address: every call asks cudaGetSymbolAddress for
+// it, with the caller's device current.  The address is not cached, because it
+// belongs to the current context's copy of the module: it changes after
+// cudaDeviceReset and differs under another context on the same device.
 static_assert((GNN_CSR_NOALLOC_MAX_EDGES + kRadixTile - 1) / kRadixTile <= 256, "histogram area too small");
 static __device__ __align__(256) unsigned char g_csr_noalloc_scratch[GNN_CSR_NOALLOC_SCRATCH_BYTES];
-static __device__ uint32_t g_csr_noalloc_err;
-
-namespace {
-constexpr int kNoallocMaxDevices = 64;
-std::mutex g_noalloc_mu;
-unsigned char* g_noalloc_scratch_dev[kNoallocMaxDevices] = {};
-uint32_t* g_noalloc_err_dev[kNoallocMaxDevices] = {};
-
-// Device addresses of the scratch array and error word on the current device.
-cudaError_t noalloc_setup(unsigned char** scratch, uint32_t** err) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kNoallocMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_scratch_dev[dev]) {
-    void* sp = nullptr;
-    void* ep = nullptr;
-    e = cudaGetSymbolAddress(&sp, g_csr_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    e = cudaGetSymbolAddress(&ep, g_csr_noalloc_err);
-    if (e != cudaSuccess) return e;
-    g_noalloc_scratch_dev[dev] = static_cast<unsigned char*>(sp);
-    g_noalloc_err_dev[dev] = static_cast<uint32_t*>(ep);
-  }
-  *scratch = g_noalloc_scratch_dev[dev];
-  *err = g_noalloc_err_dev[dev];
-  return cudaSuccess;
-}
-}  // namespace
 
 extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes, int64_t n_edges,
                                      int32_t* rowptr, int32_t* perm, int32_t* src_sorted, gnn_stream_t stream) {
-  if (n_nodes < 0 || n_nodes >= INT32_MAX || n_edges < 0 || n_edges > GNN_CSR_NOALLOC_MAX_EDGES || !rowptr)
+  if (!count_ok(n_nodes) || n_edges < 0 || n_edges > GNN_CSR_NOALLOC_MAX_EDGES || !rowptr)
     return GNN_ERR_INVALID_ARG;
   if (n_edges > 0 && (!edge_index || !perm || !src_sorted)) return GNN_ERR_INVALID_ARG;
-  unsigned char* scratch = nullptr;
-  uint32_t* err = nullptr;
-  cudaError_t ce = noalloc_setup(&scratch, &err);
+  void* sp = nullptr;                             // device address of the scratch array (current context)
+  cudaError_t ce = cudaGetSymbolAddress(&sp, g_csr_noalloc_scratch);
   if (ce != cudaSuccess) return cuda_fail(ce);
+  unsigned char* scratch = static_cast<unsigned char*>(sp);
   cudaStream_t st = (cudaStream_t)stream;
   const int N = (int)n_nodes, E = (int)n_edges;
   const int tb = 256;
   if (E == 0) {                                   // every row pointer is 0
-    csr_rowptr_kernel<<<(N + 1 + tb - 1) / tb, tb, 0, st>>>(nullptr, 0, N, rowptr);
+    csr_rowptr_kernel<<<blocks_for((int64_t)N + 1, tb), tb, 0, st>>>(nullptr, 0, N, rowptr);
     ce = cudaGetLastError();
     return ce == cudaSuccess ? GNN_OK : cuda_fail(ce);
   }
@@ -1081,12 +1083,12 @@ extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes,
   int* vals_b = vals_a + GNN_CSR_NOALLOC_MAX_EDGES;
   int* src_c = vals_b + GNN_CSR_NOALLOC_MAX_EDGES;
   int* hist = src_c + GNN_CSR_NOALLOC_MAX_EDGES;
-  csr_keys_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(edge_index, E, N, keys_a, vals_a, src_c, err);
+  csr_keys_kernel<<<blocks_for(E, tb), tb, 0, st>>>(edge_index, E, N, keys_a, vals_a, src_c, nullptr);
   int bits = 0;
   while (bits < 31 && (N >> bits) != 0) ++bits;   // keys lie in [0, N]
   if (bits == 0) bits = 1;
   const int passes = (bits + 7) / 8;
-  const int tiles = (E + kRadixTile - 1) / kRadixTile;
+  const int tiles = (int)blocks_for(E, kRadixTile);
   int *kin = keys_a, *vin = vals_a, *kout = keys_b, *vout = vals_b;
   for (int ps = 0; ps < passes; ++ps) {
     const int shift = 8 * ps;
@@ -1097,8 +1099,8 @@ extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes,
     t = vin; vin = vout; vout = t;
   }
   // sorted keys in kin; kout is free and receives the (unused) clamped destinations
-  csr_gather_kernel<<<(E + tb - 1) / tb, tb, 0, st>>>(kin, vin, src_c, E, N, perm, src_sorted, kout);
-  csr_rowptr_kernel<<<(N + 1 + tb - 1) / tb, tb, 0, st>>>(kin, E, N, rowptr);
+  csr_gather_kernel<<<blocks_for(E, tb), tb, 0, st>>>(kin, vin, src_c, E, N, perm, src_sorted, kout);
+  csr_rowptr_kernel<<<blocks_for((int64_t)N + 1, tb), tb, 0, st>>>(kin, E, N, rowptr);
   ce = cudaGetLastError();
   return ce == cudaSuccess ? GNN_OK : cuda_fail(ce);
 }

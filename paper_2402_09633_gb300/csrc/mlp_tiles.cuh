@@ -31,6 +31,7 @@
 //     quarter of the columns), reads them from tensor memory with the 16-lane
 //     shapes and does bias / gathers, LayerNorm and ReLU in registers.
 #pragma once
+#include <climits>
 #include <cstdint>
 #include <type_traits>
 #include <cuda_bf16.h>
@@ -181,28 +182,27 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     progress[0] = -1;
     progress[1] = 0;
     fence_mbar_init();
+    if (resident) {                                    // the weights are constant: load them at once
+      mbar_arrive_expect_tx(&w_full[0], (uint32_t)p.n_jobs * G::MAT_BYTES);
+      for (int j = 0; j < p.n_jobs; ++j)
+        bulk_g2s(ring + j * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[0]);
+    }
   }
   if (warp == 0) { tmem_alloc(tmem_slot, G::TMEM_COLS); tmem_relinquish(); }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // Everything above (parameter vectors, barriers, tensor memory, the resident weights) depends on
+  // no earlier kernel, so under a programmatic dependent launch it overlaps the previous kernel's
+  // exit; from here on every thread may read what that kernel wrote.
+  pdl_wait();
 
   if (warp < 4) {
     // Control warpgroup: hands registers to the worker warpgroups.
     setmaxnreg_dec<kControlRegs>();
       if (warp == 1) {
       // ------------------------------------------------ weight producer
-      if (lane == 0) {
-        if (resident) {
-          uint32_t total = 0;
-          for (int j = 0; j < p.n_jobs; ++j) total += G::MAT_BYTES;
-          mbar_arrive_expect_tx(&w_full[0], total);
-          for (int j = 0; j < p.n_jobs; ++j)
-            bulk_g2s(ring + j * G::MAT_BYTES, p.wmats + (size_t)p.job_mat[j] * p.mat_bytes, G::MAT_BYTES, &w_full[0]);
-        }
-      }
-      __syncwarp();
       if (resident && KIND == TileKind::Classifier) {
         // L2 prefetcher: while the workers are on tile pair k, warm L2 with the
         // edge-state tiles and the gathered P_s / P_d rows of pair k+1.  (The edge update
@@ -618,6 +618,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         GNN_TRACE_W(0);
         const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
         const int s1 = ok1 ? p.src_sorted[row1] : 0, d1 = ok1 ? p.dst_sorted[row1] : 0;
+        // classifier: where each row's score goes (input order) and, in the sign bit, whether an
+        // endpoint was out of range; read now so that the score store ending the tile waits on no
+        // load (measured: 0.4205 -> 0.4095 ms per launch on the full event)
+        int out0 = 0, out1 = 0;
+        if constexpr (KIND == TileKind::Classifier) {
+          if (ok0 && (lane & 3) == 0) out0 = p.perm[row0] | (p.key_sorted[row0] < p.n_nodes ? 0 : INT_MIN);
+          if (ok1 && (lane & 3) == 0) out1 = p.perm[row1] | (p.key_sorted[row1] < p.n_nodes ? 0 : INT_MIN);
+        }
         load_t16(v, p.e, row0, ok0, ok1);
         GNN_TRACE_W(1);
         put_a(v);
@@ -699,8 +707,8 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
           z1 = quad_sum(z1) + wo[H];
           if (ok && (lane & 3) == 0) {
             const float nan = __int_as_float(0x7fc00000);
-            if (ok0) p.scores[p.perm[row0]] = p.key_sorted[row0] < p.n_nodes ? 1.0f / (1.0f + __expf(-z0)) : nan;
-            if (ok1) p.scores[p.perm[row1]] = p.key_sorted[row1] < p.n_nodes ? 1.0f / (1.0f + __expf(-z1)) : nan;
+            if (ok0) p.scores[out0 & INT_MAX] = out0 >= 0 ? 1.0f / (1.0f + __expf(-z0)) : nan;
+            if (ok1) p.scores[out1 & INT_MAX] = out1 >= 0 ? 1.0f / (1.0f + __expf(-z1)) : nan;
           }
         }
       } else if constexpr (KIND == TileKind::EdgeEncoder) {
@@ -985,7 +993,10 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 // node (half a warp when H = 64): lane 4*bp + q owns the 16-byte vector q of
 // block pair bp (row-tiled T16 layout of the tile kernels), so all lanes of a
 // node run the same number of steps whatever the degree distribution, and
-// every message row is read in whole 64-byte pieces.
+// every message row is read in whole 64-byte pieces.  Blocks take the nodes
+// from the last one down: the edge update writes the messages in CSR (that is,
+// destination) order and finishes with the highest tiles, which are then still
+// in L2 when the first blocks here read them.
 template <int H>
 constexpr int agg_nodes_per_block() { return 256 / (H / 4); }
 
@@ -997,10 +1008,11 @@ __global__ void __launch_bounds__(256) aggregate_kernel(const void* __restrict__
   constexpr int LPN = H / 4;                         // lanes per node
   const SE* e = static_cast<const SE*>(e_);
   SE* agg = static_cast<SE*>(agg_);
+  pdl_wait();
   const int li = threadIdx.x % LPN;
   const int bp = li >> 2, q = li & 3;
-  const int j = blockIdx.x * agg_nodes_per_block<H>() + (int)threadIdx.x / LPN;
-  if (j >= n_nodes) return;
+  const int j = n_nodes - 1 - (blockIdx.x * agg_nodes_per_block<H>() + (int)threadIdx.x / LPN);
+  if (j < 0) return;
   const int k0 = rowptr[j], k1 = rowptr[j + 1];
   auto at = [&](int k) -> float4 {
     const SE* a = e + (((size_t)(k >> 7) * NBP + bp) * 128 + (k & 127)) * 16 + 4 * q;

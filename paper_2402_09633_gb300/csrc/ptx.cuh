@@ -264,6 +264,15 @@ __device__ __forceinline__ void setmaxnreg_dec() { asm volatile("setmaxnreg.dec.
 template <int N>
 __device__ __forceinline__ void setmaxnreg_inc() { asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N)); }
 
+// Programmatic dependent launch: the executing thread waits until every grid this one depends on has
+// completed and its memory writes are visible (it returns at once when the kernel was not launched
+// as a programmatic dependent).  Everything a kernel does before it may overlap the previous kernel,
+// so it must touch no data that kernel writes or reads.  The kernels here issue no early launch
+// trigger (griddepcontrol.launch_dependents): a dependent then launches as its predecessor's CTAs
+// exit, which hides the launch latency; measured on the full event, 6.59 -> 6.51 ms per step, while
+// triggering at the start or at the end of a tile kernel's work made it 6.83 ms.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Named barrier over `nthreads` threads (multiple of 32).
 __device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");

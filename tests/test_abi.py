@@ -59,3 +59,36 @@ def test_python_path_fails_loudly_without_library(tmp_path):
             binding.load_library(str(tmp_path / "missing.so"))
     finally:
         binding._lib = saved
+
+
+def test_counts_beyond_the_limit_rejected_before_device_work():
+    """Every count above GNN_MAX_COUNT (2^31 - 1 - 8192: the kernels round rows up to whole blocks
+    and radix tiles of up to 8192 in 32-bit arithmetic) is INVALID_ARG, checked before the context
+    is read or any device call is made.  The context pointer here is a zeroed host buffer, which a
+    call that got past its size checks would misuse."""
+    from paper_2402_09633_gb300 import binding
+    lib = binding.load_library()
+    text = open(os.path.join(ROOT, "include", "gnn.h")).read()
+    limit = int(re.search(r"#define GNN_MAX_COUNT (\d+)", text).group(1))
+    assert limit == 2 ** 31 - 1 - 8192
+    vp, i64, f32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_float
+    fake = ctypes.create_string_buffer(4096)
+    ctx, buf = ctypes.cast(fake, vp), ctypes.cast(ctypes.create_string_buffer(64), vp)
+    big, bad = limit + 1, -1
+    lib.gnn_track_labels.argtypes = [vp, vp, vp, i64, i64, f32, vp, vp]
+    lib.gnn_csr_build_noalloc.argtypes = [vp, i64, i64, vp, vp, vp, vp]
+    lib.gnn_filter_edges.argtypes = [vp, vp, vp, i64, i64, f32, vp, vp, vp, vp, vp]
+    lib.gnn_embed.argtypes = [vp, vp, i64, vp, vp]
+    lib.gnn_build_graph.argtypes = [vp, vp, ctypes.c_int, vp, i64, f32, i64, vp, vp, vp]
+    for n in (big, bad, 2 ** 31 - 1):
+        assert lib.gnn_reserve(ctx, n, 1) == -1 and lib.gnn_reserve(ctx, 1, n) == -1
+        assert lib.gnn_infer(ctx, buf, buf, n, 4, buf, None) == -1
+        assert lib.gnn_infer(ctx, buf, buf, 4, n, buf, None) == -1
+        assert lib.gnn_infer_host(ctx, buf, buf, 4, n, buf, None) == -1
+        assert lib.gnn_track_labels(ctx, buf, buf, n, 1, 0.5, buf, None) == -1
+        assert lib.gnn_track_labels(ctx, buf, buf, 4, n, 0.5, buf, None) == -1
+        assert lib.gnn_filter_edges(ctx, buf, buf, 4, n, 0.5, buf, buf, buf, buf, None) == -1
+        assert lib.gnn_embed(ctx, buf, n, buf, None) == -1
+        assert lib.gnn_build_graph(ctx, buf, 8, buf, n, 0.1, 4, buf, buf, None) == -1
+        assert lib.gnn_build_graph(ctx, buf, 8, buf, 4, 0.1, n, buf, buf, None) == -1
+        assert lib.gnn_csr_build_noalloc(buf, n, 4, buf, buf, buf, None) == -1

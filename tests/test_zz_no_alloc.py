@@ -85,3 +85,32 @@ def test_noalloc_csr_limits_and_empty_graph():
     assert lib.gnn_csr_build_noalloc(None, 10, 4, p, p, p, stream) == -1
     rc, rowptr, _, _ = _noalloc_csr(lib, dummy, 9, 0)                                  # no edges
     assert rc == 0 and rowptr.tolist() == [0] * 10
+
+
+def test_noalloc_csr_out_of_range_endpoints():
+    """Edges with an endpoint outside [0, n_nodes) sort after rowptr[n_nodes], in input order, with
+    source 0; the valid edges form the oracle's CSR of the valid subset.  The call has no error word,
+    so rowptr[n_nodes] < n_edges is the caller's only signal, and it must hold here."""
+    import torch
+    lib = _lib()
+    n = 50
+    x, ei = S.random_graph(n, 600, 3, seed=9)
+    ei = ei.copy()
+    rng = np.random.default_rng(5)
+    bad = rng.choice(ei.shape[1], 40, replace=False)
+    ei[0, bad[:10]] = -1 - rng.integers(0, 5, 10)                  # negative sources
+    ei[1, bad[10:20]] = n + rng.integers(0, 7, 10)                 # destinations past the last node
+    ei[0, bad[20:30]] = n
+    ei[1, bad[30:]] = -3
+    e = ei.shape[1]
+    rc, rowptr, perm, src = _noalloc_csr(lib, torch.from_numpy(ei).cuda(), n, e)
+    assert rc == 0
+    valid = (ei[0] >= 0) & (ei[0] < n) & (ei[1] >= 0) & (ei[1] < n)
+    ids = np.flatnonzero(valid)
+    o_rowptr, o_src, o_perm = O.csr_by_destination(ei[0, ids], ei[1, ids], n)
+    assert rowptr[n] == ids.size < e
+    np.testing.assert_array_equal(rowptr, o_rowptr)
+    np.testing.assert_array_equal(perm[:ids.size], ids[o_perm])
+    np.testing.assert_array_equal(src[:ids.size], o_src)
+    np.testing.assert_array_equal(perm[ids.size:], np.flatnonzero(~valid))
+    np.testing.assert_array_equal(src[ids.size:], 0)
