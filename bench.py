@@ -459,7 +459,7 @@ def run_gb300(args, rank: int, world: int, local: int):
         side["bf16"] = side_workload("full_bf16", max(3, min(args.steps, 50)), dev, peaks, x, ei)
         side["batch16"] = side_workload("batch16", max(3, min(args.steps, 10)), dev, peaks)
     else:
-        pipeline = run_pipeline(net, w, x, dev) if w.n_events == 1 else None
+        pipeline = run_pipeline(net, w, x, dev) if w.n_events == 1 and not args.no_side_workloads else None
         net.close()
 
     model = step_model(w)
@@ -528,7 +528,8 @@ def main():
     ap.add_argument("--workload", choices=tuple(S.WORKLOADS), default="full")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-side-workloads", action="store_true",
-                    help="skip the bf16-model and 16-event-batch sub-objects (timed after the headline)")
+                    help="skip what is timed after the headline: the pipeline stages and the bf16-model and "
+                         "16-event-batch sub-objects")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))

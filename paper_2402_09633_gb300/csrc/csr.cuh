@@ -55,28 +55,54 @@ __global__ void radix_count_kernel(const int* __restrict__ keys, int n, int shif
 
 // Scatter offsets of one radix pass, in place: hist[tile * 256 + d] becomes the
 // number of keys with a smaller digit (all tiles) plus those with digit d in
-// earlier tiles.  One block of 256 threads; thread d walks its digit's column
-// (reads are coalesced across threads), then the 256 digit totals are scanned.
-__global__ void __launch_bounds__(256) radix_offsets_kernel(int* __restrict__ hist, int n_tiles) {
+// earlier tiles.  One block of kOffsetsThreads: thread (part, d) owns digit d
+// over one contiguous quarter of the tiles (reads coalesced across digits) and
+// keeps kOffsetsBatch loads in flight; the quarters' sums and the 256 digit
+// totals are combined in shared memory.  (A single thread per digit walking
+// every tile with one dependent load at a time took 23 us per pass.)
+constexpr int kOffsetsThreads = 1024;
+constexpr int kOffsetsParts = kOffsetsThreads / 256;
+constexpr int kOffsetsBatch = 16;
+__global__ void __launch_bounds__(kOffsetsThreads) radix_offsets_kernel(int* __restrict__ hist, int n_tiles) {
   pdl_wait();
+  __shared__ int part_sum[kOffsetsParts][256];
   __shared__ int tot[256];
-  const int d = threadIdx.x;
-  int run = 0;
-  for (int t = 0; t < n_tiles; ++t) {
-    const int v = hist[t * 256 + d];
-    hist[t * 256 + d] = run;
-    run += v;
+  const int d = threadIdx.x & 255, part = threadIdx.x >> 8;
+  const int per = (n_tiles + kOffsetsParts - 1) / kOffsetsParts;
+  const int t0 = part * per, t1 = min(n_tiles, t0 + per);
+  int sum = 0;
+  for (int t = t0; t < t1; t += kOffsetsBatch) {            // pass 1: this quarter's count of digit d
+    int v[kOffsetsBatch];
+#pragma unroll
+    for (int i = 0; i < kOffsetsBatch; ++i) v[i] = t + i < t1 ? hist[(t + i) * 256 + d] : 0;
+#pragma unroll
+    for (int i = 0; i < kOffsetsBatch; ++i) sum += v[i];
   }
-  tot[d] = run;
+  part_sum[part][d] = sum;
   __syncthreads();
-  for (int off = 1; off < 256; off <<= 1) {       // inclusive scan of the digit totals
-    const int v = d >= off ? tot[d - off] : 0;
+  if (part == 0) {
+    int all = 0;
+#pragma unroll
+    for (int k = 0; k < kOffsetsParts; ++k) all += part_sum[k][d];
+    tot[d] = all;
+  }
+  __syncthreads();
+  for (int off = 1; off < 256; off <<= 1) {                  // inclusive scan of the digit totals
+    const int v = (part == 0 && d >= off) ? tot[d - off] : 0;
     __syncthreads();
-    tot[d] += v;
+    if (part == 0) tot[d] += v;
     __syncthreads();
   }
-  const int base = tot[d] - run;                  // exclusive
-  for (int t = 0; t < n_tiles; ++t) hist[t * 256 + d] += base;
+  int run = d > 0 ? tot[d - 1] : 0;                          // keys with a smaller digit
+  for (int k = 0; k < part; ++k) run += part_sum[k][d];      // digit d in earlier quarters
+  for (int t = t0; t < t1; t += kOffsetsBatch) {            // pass 2: exclusive offsets
+    int v[kOffsetsBatch];
+#pragma unroll
+    for (int i = 0; i < kOffsetsBatch; ++i) v[i] = t + i < t1 ? hist[(t + i) * 256 + d] : 0;
+#pragma unroll
+    for (int i = 0; i < kOffsetsBatch; ++i)
+      if (t + i < t1) { hist[(t + i) * 256 + d] = run; run += v[i]; }
+  }
 }
 
 // Stable scatter of one radix pass.  Elements of a tile are ranked in input

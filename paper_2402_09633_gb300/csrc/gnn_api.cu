@@ -396,7 +396,7 @@ int build_csr(gnn_ctx* c, const int32_t* ei, int N, int E, cudaStream_t st) {
   for (int ps = 0; ps < passes; ++ps) {
     const int shift = 8 * ps;
     chk(launch_pdl(radix_count_kernel, tiles, kRadixThreads, 0, st, (const int*)kin, E, shift, tiles, c->hist));
-    chk(launch_pdl(radix_offsets_kernel, 1, 256, 0, st, c->hist, tiles));
+    chk(launch_pdl(radix_offsets_kernel, 1, kOffsetsThreads, 0, st, c->hist, tiles));
     chk(launch_pdl(radix_scatter_kernel, tiles, kRadixThreads, 0, st, (const int*)kin, (const int*)vin, kout, vout, E,
                    shift, tiles, (const int*)c->hist));
     int* t = kin; kin = kout; kout = t;
@@ -894,7 +894,7 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   int *kin = keys_a, *vin = vals_a, *kout = keys_b, *vout = vals_b;
   for (int ps = 0; ps < passes; ++ps) {
     radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, N, 8 * ps, tiles, hist);
-    radix_offsets_kernel<<<1, 256, 0, st>>>(hist, tiles);
+    radix_offsets_kernel<<<1, kOffsetsThreads, 0, st>>>(hist, tiles);
     radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, N, 8 * ps, tiles, hist);
     int* t = kin; kin = kout; kout = t;
     t = vin; vin = vout; vout = t;
@@ -1093,7 +1093,7 @@ extern "C" int gnn_csr_build_noalloc(const int32_t* edge_index, int64_t n_nodes,
   for (int ps = 0; ps < passes; ++ps) {
     const int shift = 8 * ps;
     radix_count_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, E, shift, tiles, hist);
-    radix_offsets_kernel<<<1, 256, 0, st>>>(hist, tiles);
+    radix_offsets_kernel<<<1, kOffsetsThreads, 0, st>>>(hist, tiles);
     radix_scatter_kernel<<<tiles, kRadixThreads, 0, st>>>(kin, vin, kout, vout, E, shift, tiles, hist);
     int* t = kin; kin = kout; kout = t;
     t = vin; vin = vout; vout = t;
