@@ -41,6 +41,7 @@ METRIC = "GNN inference edges/sec and events/sec (300k-node/1M-edge) on 1 GB300;
 UNIT = "edges/s"
 L2_FLUSH_BYTES = 256 << 20          # > 2x the 129 MB L2, written between timed steps
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+NOMINAL_HBM_GBS = 7900.0       # GB300 HBM3e datasheet bandwidth; fractions against it are a second line
 
 
 def load_peaks():
@@ -53,6 +54,16 @@ def load_peaks():
 
 
 # ------------------------------------------------------------------ traffic model
+def step_roofline(model, peaks, mean_ms: float, **extra):
+    """Step-level roofline: the algorithmic bytes and flops of one step against the measured
+    peaks (the headline fraction), and the bytes against the nominal HBM bandwidth."""
+    t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9), model["flops"] / (peaks["bf16_tflops"] * 1e12))
+    t_nom_ms = 1e3 * max(model["bytes"] / (NOMINAL_HBM_GBS * 1e9), model["flops"] / (peaks["bf16_tflops"] * 1e12))
+    return {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms, "bytes_alg": model["bytes"],
+            "flops_alg": model["flops"], "t_roof_nominal_hbm_ms": t_nom_ms, "frac_of_nominal_hbm": t_nom_ms / mean_ms,
+            **extra}
+
+
 def step_model(w: S.Workload):
     """Algorithmic bytes and flops of one step (whole path) and of the two iteration kernels."""
     m, ev = w.model, w.event
@@ -364,13 +375,11 @@ def side_workload(name: str, steps: int, dev, peaks, x_dev=None, ei_dev=None):
     net.close()
     mean_ms = sum(ms) / len(ms)
     model = step_model(w)
-    t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9), model["flops"] / (peaks["bf16_tflops"] * 1e12))
     out = {"workload": name, "description": w.description, "n_nodes": N, "n_edges": E,
            "steps": steps, "ms_per_step": mean_ms, "edges_per_s": E / (mean_ms * 1e-3),
            "events_per_s": w.n_events / (mean_ms * 1e-3),
            "dtype": "bf16->f32" if w.model.precision == S.PRECISION_BF16 else "bf16x3->f32",
-           "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms, "bytes_alg": model["bytes"],
-                             "flops_alg": model["flops"], "bytes_per_activation": 2 if w.model.precision else 4},
+           "step_roofline": step_roofline(model, peaks, mean_ms, bytes_per_activation=2 if w.model.precision else 4),
            "kernels": {g: v["ms_per_launch"] for g, v in groups.items()}, "device_status": status}
     if w.model.precision == S.PRECISION_BF16:
         out["tolerance"] = ("stated 1e-2 max on logits is not met: the GPU's max logit error against the "
@@ -472,6 +481,7 @@ def run_gb300(args, rank: int, world: int, local: int):
         achieved = dom_model["bytes"] / dom_avg_s / 1e9
         roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"],
                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                    "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS,
                     "traffic": profiled_traffic(dom, w.model.precision == S.PRECISION_BF16),
                     "peak_source": f"{peak_src} (hbm_gbs, copy burst) -- of {peak_src}",
                     "bytes_per_launch": dom_model["bytes"], "avg_launch_ms": dom_avg_s * 1e3,
@@ -479,8 +489,6 @@ def run_gb300(args, rank: int, world: int, local: int):
                                      f"{split_steps} profiled steps after the headline",
                     "tensor_tflops_executed": (1 if w.model.precision == S.PRECISION_BF16 else 3)
                                               * dom_model["flops"] / dom_avg_s / 1e12}
-    t_roof_ms = 1e3 * max(model["bytes"] / (peaks["hbm_gbs"] * 1e9),
-                          model["flops"] / (peaks["bf16_tflops"] * 1e12))
     launches_per_step = sum(v["launches"] for v in kernels_only.values()) / split_steps
 
     cpu = None
@@ -499,8 +507,7 @@ def run_gb300(args, rank: int, world: int, local: int):
             "config": workload_config(w),
             "events_per_s": value / E * w.n_events,                 # every rank scores events of E edges
             "roofline": roofline,
-            "step_roofline": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / mean_ms,
-                              "bytes_alg": model["bytes"], "flops_alg": model["flops"]},
+            "step_roofline": step_roofline(model, peaks, mean_ms),
             "kernels": groups,
             "kernels_pass": {"steps": split_steps, "ms_per_step_with_events": profiled_ms},
             **side,

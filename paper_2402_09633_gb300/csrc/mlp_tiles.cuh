@@ -165,8 +165,8 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
   uint64_t* w_empty = bars + 4 + G::STAGES;          // [STAGES]  both slots' MMAs on a stage completed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * G::STAGES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  volatile int* progress = abort_flag + 1;          // [0] tile pair slot 0's workers are on (classifier L2 prefetch pacing)
-                                                    // [1] slot 1 may start (edge kernels: the slots run out of phase)
+  volatile int* slot1_go = abort_flag + 1;          // slot 1 may start (edge kernels: the slots run out of phase)
+  volatile int* cur_pair = abort_flag + 2;          // tile pair slot 0 is on (written only, see the worker loop)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -179,8 +179,8 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     mbar_init(&d_full[0], 1); mbar_init(&d_full[1], 1);
     for (int s = 0; s < G::STAGES; ++s) { mbar_init(&w_full[s], 1); mbar_init(&w_empty[s], 2); }
     *abort_flag = 0;
-    progress[0] = -1;
-    progress[1] = 0;
+    *slot1_go = 0;
+    *cur_pair = -1;
     fence_mbar_init();
     if (resident) {                                    // the weights are constant: load them at once
       mbar_arrive_expect_tx(&w_full[0], (uint32_t)p.n_jobs * G::MAT_BYTES);
@@ -203,34 +203,6 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
     setmaxnreg_dec<kControlRegs>();
       if (warp == 1) {
       // ------------------------------------------------ weight producer
-      if (resident && KIND == TileKind::Classifier) {
-        // L2 prefetcher: while the workers are on tile pair k, warm L2 with the
-        // edge-state tiles and the gathered P_s / P_d rows of pair k+1.  (The edge update
-        // prefetches from its workers instead: this warp made it 4 % slower, with only the
-        // gathered rows 7 %, with the rows paced to its layer-2 point 29 %.)
-        const uint64_t t0 = global_timer_ns();
-        for (int pair = blockIdx.x; pair < n_pairs && !*abort_flag; pair += gridDim.x) {
-          const int prev = pair - (int)gridDim.x;
-          for (uint32_t it = 0; prev >= 0 && progress[0] < prev; ++it) {    // bounded: gives up silently
-            if (*abort_flag || ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs)) break;
-            __nanosleep(200);
-          }
-          for (int s = 0; s < 2; ++s) {
-            const int tile = 2 * pair + s;
-            if (tile >= p.n_tiles) break;
-            if (lane == 0)
-              prefetch_l2_bulk(static_cast<const SE*>(p.e) + (size_t)tile * kTileRows * H, kTileRows * H * sizeof(SE));
-#pragma unroll
-            for (int i = 0; i < kTileRows / 32; ++i) {
-              const int row = tile * kTileRows + i * 32 + lane;
-              if (row < p.n_rows) {
-                prefetch_l2_bulk(p.ps + (size_t)p.src_sorted[row] * H, H * 4);
-                prefetch_l2_bulk(p.pd + (size_t)p.dst_sorted[row] * H, H * 4);
-              }
-            }
-          }
-        }
-      }
       if (resident && lane == 0) drain_wait(&w_full[0], 0);     // the resident weights have landed
       if (!resident && lane == 0) {
         {
@@ -600,20 +572,24 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
 
       if constexpr (KIND == TileKind::EdgeUpdate || KIND == TileKind::Classifier) {
         // vec layout: [gamma1, beta1, (b_l, gamma_l, beta_l) for l = 2..L, (w_o, b_o)]
-        if (slot == 0 && ws == 0 && lane == 0) progress[0] = pair;   // paces the classifier's L2 prefetcher
         // The two slots run out of phase: slot 1 starts once slot 0 has released the last MMA of
         // its first tile, so that one slot's tile change (store, next loads) overlaps the other
         // slot's MMAs instead of leaving the tensor core idle.  Bounded: it starts anyway after
         // the wait limit.
         if (slot == 1 && pair == (int)blockIdx.x) {
           const uint64_t t0 = global_timer_ns();
-          for (uint32_t it = 0; progress[1] == 0; ++it) {
+          for (uint32_t it = 0; *slot1_go == 0; ++it) {
             if (*abort_flag || ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs)) break;
             __nanosleep(64);
           }
         }
+        // Edge update: slot 0 records its tile pair.  Nothing reads the word; the store stays
+        // because without it ptxas allocates the fp32 edge update's worker registers differently
+        // and spills 28 B (measured: 0.391 -> 0.404 ms per launch).  The classifier is faster
+        // without it (0.384 -> 0.373 ms).
+        if (KIND == TileKind::EdgeUpdate && slot == 0 && ws == 0 && lane == 0) *cur_pair = pair;
         auto release_slot1 = [&]() {
-          if (slot == 0 && pair == (int)blockIdx.x && j == L && ws == 0 && lane == 0) progress[1] = 1;
+          if (slot == 0 && pair == (int)blockIdx.x && j == L && ws == 0 && lane == 0) *slot1_go = 1;
         };
         GNN_TRACE_W(0);
         const int s0 = ok0 ? p.src_sorted[row0] : 0, d0 = ok0 ? p.dst_sorted[row0] : 0;
@@ -671,11 +647,14 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         for (int l = 2; l <= L; ++l) {
           wait_job();
           GNN_TRACE_W(5 + 2 * (l - 1));
-          if (KIND == TileKind::EdgeUpdate && l == 2 && ws == 0 && lane == 0) {
+          if ((KIND == TileKind::EdgeUpdate || (KIND == TileKind::Classifier && !BF)) && l == 2 && ws == 0 &&
+              lane == 0) {
             // Warm L2 with this slot's next edge-state tile, a few microseconds before its load
             // (bulk prefetch: the copy engine, not the SM's load path).  Measured on the full
-            // event: 0.484 -> 0.395 ms per launch; issued after layer 1 (0.420) or layer 3 (0.412)
-            // it helps less.
+            // event: edge update 0.484 -> 0.395 ms per launch; issued after layer 1 (0.420) or
+            // layer 3 (0.412) it helps less.  Classifier: 0.376 ms against 0.394 without any
+            // prefetch and 0.416 with a warp prefetching the next pair's tiles and gathered rows;
+            // the bf16 classifier is fastest without prefetch (0.331, 0.342 with this one).
             const int nt = tile + 2 * (int)gridDim.x;
             if (nt < p.n_tiles)
               prefetch_l2_bulk(static_cast<const SE*>(p.e) + (size_t)nt * kTileRows * H, kTileRows * H * sizeof(SE));

@@ -90,6 +90,28 @@ def test_edge_cases_degenerate_graphs():
     assert s[0] == s[1] == s[2]
 
 
+def test_hub_nodes_long_segments():
+    """Two hubs: node 17 receives 60 % of the edges (one CSR segment across ~140 edge tiles) and
+    the last node 20 % (the first node the aggregation blocks reach).  Long segments, sums that
+    cross many tiles, and a CSR dominated by two keys; CSR bit-exact, scores against the oracle."""
+    import torch
+    n, e = 3000, 30000
+    cfg = S.ModelConfig(3, 2, 128, 2, 3)
+    W = S.init_weights(cfg, 5)
+    x, ei = S.random_graph(n, e, 3, 21)
+    k = np.random.default_rng(22).permutation(e)
+    ei[1, k[:18000]] = 17
+    ei[1, k[18000:24000]] = n - 1
+    s, rc, net = run_gpu(cfg, W, x, ei, return_net=True)
+    assert rc == 0
+    rowptr, src_sorted, perm = O.csr_by_destination(ei[0], ei[1], n)
+    np.testing.assert_array_equal(net.debug_copy(0, (n + 1,), torch.int32).cpu().numpy(), rowptr)
+    np.testing.assert_array_equal(net.debug_copy(1, (e,), torch.int32).cpu().numpy(), perm)
+    net.close()
+    assert rowptr[18] - rowptr[17] >= 18000 and rowptr[n] - rowptr[n - 1] >= 6000
+    check_parity(s, W, x, ei, cfg.n_iters)
+
+
 def test_empty_edge_list_is_noop():
     import torch
     from paper_2402_09633_gb300 import InteractionNetwork
