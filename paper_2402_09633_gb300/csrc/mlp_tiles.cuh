@@ -724,18 +724,35 @@ __global__ void __launch_bounds__(kThreads, 1) mlp_tile_kernel(const TileParams 
         ln_relu(v, vb + H, vb + 2 * H);
         put_a(v);
         arrive_a(j, seq); next_job();
+        // Deeper layers: the fp32 model streams its epilogues, the bf16 model keeps the row in
+        // registers (measured per launch, streamed / register form: fp32 0.285 / 0.293 ms, bf16
+        // 0.232 / 0.219 ms).
         for (int l = 2; l < L; ++l) {
           wait_job();
           const float* vl = vb + 3 * (l - 1) * H;
-          ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { put_a_chunk(k, t); });
-          tmem_st_wait();
+          if constexpr (BF) {
+            load_d(v);
+            add_vec(v, vl);
+            ln_relu(v, vl + H, vl + 2 * H);
+            put_a(v);
+          } else {
+            ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { put_a_chunk(k, t); });
+            tmem_st_wait();
+          }
           arrive_a(j, seq); next_job();
         }
         wait_job();
         {
           const float* vl = vb + 3 * (L - 1) * H;
           const bool w0 = ok && ok0, w1 = ok && ok1;
-          ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { store_t16_chunk(p.e, row0, w0, w1, k, t); });
+          if constexpr (BF) {
+            load_d(v);
+            add_vec(v, vl);
+            ln_relu(v, vl + H, vl + 2 * H);
+            store_t16(p.e, row0, w0, w1, v);
+          } else {
+            ln_stream(vl, vl + H, vl + 2 * H, [&](int k, const float* t) { store_t16_chunk(p.e, row0, w0, w1, k, t); });
+          }
         }
       } else if constexpr (KIND == TileKind::Embed) {
         // vec layout: [W1^T (F_n x H), (b_l, gamma_l, beta_l) for l = 1..L, W_out rows (D x H), b_out (D)]
