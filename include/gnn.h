@@ -168,8 +168,9 @@ int gnn_infer_host(gnn_ctx* ctx, const float* node_feats, const int32_t* edge_in
  * count (saturated at INT32_MAX), and gnn_status reports GNN_ERR_CAPACITY: call again with room
  * for that many.  The order
  * of the edges is deterministic.  Uses a scratch buffer of the context (grown on demand,
- * synchronous then).  Errors: INVALID_ARG (radius <= 0, emb_dim out of range, null pointer, bad
- * sizes), OOM, CUDA.
+ * synchronous then): besides the sorted copies, 128 bytes per hit for the partner chains the
+ * counting pass keeps (see gnn_debug_graph_pool).  Errors: INVALID_ARG (radius <= 0, emb_dim out
+ * of range, null pointer, bad sizes), OOM, CUDA.
  */
 int gnn_embed_load(gnn_ctx* ctx, const void* weights_host, size_t weights_bytes);
 int gnn_embed(gnn_ctx* ctx, const float* node_feats, int64_t n_nodes, float* embedding, gnn_stream_t stream);
@@ -288,6 +289,17 @@ int gnn_debug_copy(gnn_ctx* ctx, int which, void* dst, size_t bytes, gnn_stream_
  */
 int gnn_debug_fail_allocs(int n);
 int gnn_debug_wait_timeout(gnn_ctx* ctx, int64_t limit_ns, gnn_stream_t stream);
+
+/*
+ * gnn_debug_graph_pool -- test hook for gnn_build_graph (no paper counterpart).  The counting pass
+ * keeps every hit's partners in a chain of 15-entry chunks, the hit's own first chunk plus chunks
+ * from a pool, and the writing pass copies them; a hit whose chain could not grow because the pool
+ * was used up is searched again instead, with the same result.  This sets the pool size in chunks
+ * for later calls on this context (0: every hit with more than 15 partners takes the search-again
+ * path); a negative value restores the default of one pool chunk per hit.  Errors: INVALID_ARG
+ * (null context).
+ */
+int gnn_debug_graph_pool(gnn_ctx* ctx, int64_t chunks);
 
 /*
  * gnn_csr_build_noalloc -- the destination-keyed CSR of an edge list, built

@@ -75,6 +75,7 @@ struct gnn_ctx {
   float embed_eps = 0.f;
   int* aux = nullptr;
   size_t aux_ints = 0;
+  int64_t graph_pool = -1;             // graph building: pool chunks for partner chains (-1: one per hit)
   uint32_t* d_err = nullptr;
   // workspace
   void* ws = nullptr;
@@ -866,10 +867,16 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   for (int k = 0; k < K; ++k) n_cells *= grid;
   const int tiles = (int)blocks_for(N, kRadixTile);
   const int chunks = (emb_dim + 3) / 4;                   // float4 chunks per sorted embedding
-  // scratch: emb_s [N, 4 * chunks] (first, 16-byte aligned), r_s, keys/vals (two buffers each),
-  // per-hit counts, per-block sums, radix histograms, cell starts
+  // partner chains kept by the counting pass: one first chunk per hit, pool chunks after them (a hit
+  // whose chain cannot grow is searched again by the writing pass)
+  const int64_t pool64 = ctx->graph_pool >= 0 ? ctx->graph_pool : (int64_t)N;
+  const int pool = (int)(pool64 < (int64_t)INT_MAX - N ? pool64 : (int64_t)INT_MAX - N);
+  // scratch: emb_s [N, 4 * chunks] (first, 16-byte aligned), partner chunks, r_s, keys/vals (two
+  // buffers each), per-hit counts, per-block sums, radix histograms, cell starts, the pool counter
   const int nb = (int)blocks_for(N, tb);
-  const size_t need = 4 * (size_t)chunks * N + 6 * (size_t)N + (size_t)nb + 256 * (size_t)tiles + (size_t)n_cells + 1;
+  const size_t chain_ints = ((size_t)N + (size_t)pool) * kFrnnChunk;
+  const size_t need = 4 * (size_t)chunks * N + chain_ints + 6 * (size_t)N + (size_t)nb + 256 * (size_t)tiles +
+                      (size_t)n_cells + 2;
   if (need > ctx->aux_ints) {
     if (ctx->aux) { cudaStreamSynchronize(st); cudaFree(ctx->aux); ctx->aux = nullptr; ctx->aux_ints = 0; }
     const cudaError_t err = dev_alloc((void**)&ctx->aux, need * sizeof(int));
@@ -877,7 +884,8 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
     ctx->aux_ints = need;
   }
   float4* emb_s = (float4*)ctx->aux;
-  float* r_s = (float*)(ctx->aux + 4 * (size_t)chunks * N);
+  int* chains = (int*)(ctx->aux + 4 * (size_t)chunks * N);
+  float* r_s = (float*)(chains + chain_ints);
   int* keys_a = (int*)(r_s + N);
   int* keys_b = keys_a + N;
   int* vals_a = keys_b + N;
@@ -886,6 +894,7 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   int* block_sums = counts + N;
   int* hist = block_sums + nb;
   int* cell_start = hist + 256 * (size_t)tiles;
+  int* next_chunk = cell_start + n_cells + 1;
   if (K == 4) frnn_cell_kernel<4><<<nb, tb, 0, st>>>(embedding, N, emb_dim, grid, keys_a, vals_a);
   else frnn_cell_kernel<3><<<nb, tb, 0, st>>>(embedding, N, emb_dim, grid, keys_a, vals_a);
   int bits = 0;
@@ -900,6 +909,10 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
     t = vin; vin = vout; vout = t;
   }
   csr_rowptr_kernel<<<blocks_for((int64_t)n_cells + 1, tb), tb, 0, st>>>(kin, N, n_cells, cell_start);
+  {
+    const cudaError_t e0 = cudaMemsetAsync(next_chunk, 0, sizeof(int), st);
+    if (e0 != cudaSuccess) return cuda_fail(e0);
+  }
   const float r2 = radius * radius;
   const int xs = ctx->cfg.n_node_feat;
   const int sb = (int)blocks_for(N, kScanBlock);
@@ -909,13 +922,15 @@ int gnn_build_graph(gnn_ctx* ctx, const float* embedding, int emb_dim, const flo
   case CH * 8 + KK:                                                                                              \
     frnn_gather_kernel<CH><<<nb, tb, 0, st>>>(embedding, node_feats, xs, N, emb_dim, vin, emb_s, r_s);         \
     frnn_pairs_kernel<CH, KK><<<pb, kFrnnPairsThreads, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, \
-                                                                0, counts, nullptr, 0, nullptr, ctx->d_err);     \
+                                                                0, counts, nullptr, 0, nullptr, chains,          \
+                                                                next_chunk, pool, ctx->d_err);                   \
     scan_reduce_kernel<<<sb, kScanBlock, 0, st>>>(counts, N, block_sums);                                      \
     compact_scan_kernel<<<1, 1024, 0, st>>>(block_sums, sb, n_edges);                                            \
     scan_apply_kernel<<<sb, kScanBlock, 0, st>>>(counts, N, block_sums);                                       \
     frnn_pairs_kernel<CH, KK><<<pb, kFrnnPairsThreads, 0, st>>>(emb_s, r_s, N, r2, grid, kin, vin, cell_start, \
                                                                 1, counts, n_edges, (int)max_edges, edge_index,  \
-                                                                ctx->d_err);                                     \
+                                                                chains, next_chunk, pool, ctx->d_err);           \
+    frnn_copy_kernel<<<nb, tb, 0, st>>>(r_s, N, vin, counts, n_edges, (int)max_edges, chains, edge_index);      \
     break;
     GNN_FRNN_CASE(1, 3)
     GNN_FRNN_CASE(2, 3)
@@ -956,6 +971,12 @@ int gnn_trace_read(gnn_ctx* ctx, unsigned long long* host) {
 int gnn_debug_fail_allocs(int n) {
   if (n < 0) return GNN_ERR_INVALID_ARG;
   g_fail_allocs.store(n);
+  return GNN_OK;
+}
+
+int gnn_debug_graph_pool(gnn_ctx* ctx, int64_t chunks) {
+  if (!ctx) return GNN_ERR_INVALID_ARG;
+  ctx->graph_pool = chunks < 0 ? -1 : chunks;
   return GNN_OK;
 }
 

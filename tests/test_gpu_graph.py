@@ -98,6 +98,37 @@ def test_radius_graph_other_embedding_widths(dim):
     net.close()
 
 
+def test_partner_chains_and_search_again_agree():
+    """The counting pass keeps each hit's partners in chains of 15-entry chunks that the writing pass
+    copies; a hit whose chain could not grow (pool used up) is searched again.  At a radius giving
+    about 40 neighbours per hit (chains of several chunks), the default pool, an empty pool and a
+    pool that runs out part-way give byte-identical edge lists, equal to the oracle's edge set."""
+    import ctypes
+    import torch
+    cfg = S.ModelConfig(12, 2, 64, 2, 2)
+    net, _, _ = _net(cfg)
+    n = 8000
+    x, _ = S.generate_event(S.EventSpec(n, 9, "powerlaw", 0.02, n_edges=3 * n), 4)
+    xs = torch.from_numpy(x).cuda()
+    emb = net.embed(xs)
+    e_np = emb.cpu().numpy()
+    radius = _radius_for(e_np, 40)
+    net.lib.gnn_debug_graph_pool.argtypes = [ctypes.c_void_p, ctypes.c_int64]
+    net.lib.gnn_debug_graph_pool.restype = ctypes.c_int
+    outs = []
+    for pool in (-1, 0, 100):
+        assert net.lib.gnn_debug_graph_pool(net.handle, pool) == 0
+        ei, m = net.build_graph(emb, xs, radius, max_edges=100 * n)
+        assert net.status() == 0
+        outs.append(ei.cpu().numpy().tobytes())
+    assert outs[0] == outs[1] == outs[2]
+    got = _sorted_edges(np.frombuffer(outs[0], np.int32).reshape(2, -1))
+    assert got.shape[0] > 15 * n                       # more than one chunk per hit on average
+    np.testing.assert_array_equal(got, _oracle_graph(e_np, x[:, 0], radius))
+    assert net.lib.gnn_debug_graph_pool(None, 0) == -1
+    net.close()
+
+
 def test_radius_graph_full_event_sampled():
     """300k hits: the edges of 400 sampled hits against a brute-force search over every hit, and
     the properties every edge list must have (no self-loops, no duplicates, oriented by r)."""
