@@ -43,6 +43,38 @@ def test_batch16_events_equal_their_standalone_scores():
     net.close()
 
 
+def test_64_copies_interleaved_equal_standalone():
+    """Size well beyond the 16-event batch: 64 copies of the full event as one block-diagonal graph
+    (19.2M nodes, 64M edges, about 75 GB of state), their edges interleaved in blocks of 1000 by a
+    seeded random merge that keeps each copy's own edge order.  The CSR sort is stable, so every node
+    sums its messages in the same order as in the standalone event: each copy's scores equal the
+    standalone scores bit for bit."""
+    import torch
+    from paper_2402_09633_gb300 import InteractionNetwork
+    w = S.WORKLOADS["full"]
+    W = S.init_weights(w.model, 0)
+    x, ei = S.generate_event(w.event, 0)
+    N, E, C, B = x.shape[0], ei.shape[1], 64, 1000
+    assert E % B == 0
+    labels = np.repeat(np.arange(C, dtype=np.int32), E // B)
+    np.random.default_rng(5).shuffle(labels)
+    blocks = np.argsort(labels, kind="stable").reshape(C, E // B)   # copy k's blocks land there, in order
+    slots = (blocks[:, :, None] * B + np.arange(B)).reshape(C, E)    # slots[k] = where copy k's edges go
+    eib = np.empty((2, C * E // B, B), np.int32)
+    for k in range(C):
+        eib[:, blocks[k], :] = (ei + np.int32(k * N)).reshape(2, E // B, B)
+    eib = eib.reshape(2, C * E)
+    xb = np.tile(x, (C, 1))
+    net = InteractionNetwork(w.model, S.pack_blob(w.model, W))
+    s1 = net.infer(torch.from_numpy(x).cuda(), torch.from_numpy(ei).cuda()).cpu().numpy()
+    sb = net.infer(torch.from_numpy(xb).cuda(), torch.from_numpy(eib).cuda()).cpu().numpy()
+    assert net.status() == 0
+    net.close()
+    for k in (0, 1, 31, 63):
+        assert sb[slots[k]].tobytes() == s1.tobytes(), f"copy {k} differs inside the batch"
+    assert np.array_equal(sb[slots].reshape(C, E), np.broadcast_to(s1, (C, E)))
+
+
 def test_small_batch_parity_against_oracle():
     w = S.WORKLOADS["full"]
     W = S.init_weights(w.model, 0)
