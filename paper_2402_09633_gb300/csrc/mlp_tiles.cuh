@@ -24,12 +24,13 @@
 //   * control warpgroup (warps 0-3): warp 0 issues the MMAs of whichever slot
 //     has published its next A operand (one thread, 24 tcgen05.mma per layer)
 //     and commits them to the slot's mbarrier; warp 1 loads the weights with
-//     bulk copies (all at once, or streamed through a ring of stages) and
-//     warms L2 with the next tile pair's rows;
+//     bulk copies (all at once, or streamed through a ring of stages);
 //   * worker warpgroups (warps 4-19), eight warps per slot: a worker warp owns
 //     16 rows of a tile; a quad of threads shares two rows (each thread a
 //     quarter of the columns), reads them from tensor memory with the 16-lane
-//     shapes and does bias / gathers, LayerNorm and ReLU in registers.
+//     shapes and does bias / gathers, LayerNorm and ReLU in registers; one
+//     worker thread per slot warms L2 (bulk prefetch) with the slot's next
+//     tile a few microseconds before it is loaded.
 #pragma once
 #include <climits>
 #include <cstdint>
